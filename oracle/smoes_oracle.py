@@ -1,0 +1,391 @@
+"""Plain fp64 CPU oracle of the SMoES modality-guided router (test infrastructure).
+
+This module is TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may import it. The product path (the CUDA library behind
+``include/smoes.h`` and its Python binding) never calls it, and it shares no code, header,
+table or helper with that path.
+
+Every function follows the paper ("Soft Modality-Guided Expert Specialization in MoE-VLMs")
+step by step, in float64, with numpy primitives (matmul, sort, log/exp) only. Where the paper
+is silent the reading used is stated in the docstring; the same readings are listed in
+the design doc.
+
+Conventions
+-----------
+* Modality index m: 0 = vision, 1 = text (columns of the score matrix M [T, 2]).
+* Samples are contiguous token ranges given by ``sample_offsets`` [B+1].
+* ``expert_bin`` [E] maps each routed expert to its bin; every bin holds N_B = E / n_bins
+  experts.
+* Natural logarithms throughout.
+
+Pins (what fixes this oracle independently of itself) live in ``tests/test_oracle_*.py``.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+# A modality whose total soft mass in a sample is at or below this value is treated as absent
+# from the sample (eq. 12 would be 0/0). Reading: its bin-averaged gating scores are 0.
+MASS_EPS = 1e-12
+
+
+def _f64(a):
+    return np.asarray(a, dtype=np.float64)
+
+
+# --------------------------------------------------------------------------------------------
+# Soft modality scores (Sec. 3.2)
+# --------------------------------------------------------------------------------------------
+
+def gaussian_log_likelihood(X, mu, var):
+    """Diagonal-Gaussian log-likelihood of every token under each modality, eq. (8).
+
+    LL[j, m] = -1/2 * sum_d ( log var[m, d] + (x[j, d] - mu[m, d])^2 / var[m, d] ).
+
+    X [T, d]; mu, var [2, d] (row 0 vision, row 1 text) -> LL [T, 2].
+    """
+    X, mu, var = _f64(X), _f64(mu), _f64(var)
+    T = X.shape[0]
+    LL = np.empty((T, 2))
+    for m in range(2):
+        LL[:, m] = -0.5 * np.sum(np.log(var[m])[None, :] + (X - mu[m][None, :]) ** 2 / var[m][None, :],
+                                 axis=1)
+    return LL
+
+
+def gaussian_score(X, mu, var, tau):
+    """Gaussian-statistics soft modality score, eq. (9): softmax over modalities of LL / tau.
+
+    Returns M [T, 2] with M[:, 0] = vision score and M[:, 1] = text score.
+    The paper's default temperature is tau = 0.5 * D with D the hidden size (Sec. 4.1).
+    """
+    LL = gaussian_log_likelihood(X, mu, var) / float(tau)
+    LL = LL - LL.max(axis=1, keepdims=True)
+    e = np.exp(LL)
+    return e / e.sum(axis=1, keepdims=True)
+
+
+def attention_vision_mass(Q, K, m_keys, sm_scale, causal=True, key_bias=None, queries=None):
+    """Attention-accumulated vision score, eqs. (2)-(3).
+
+    For sequence b and query j the aggregated score is
+        Mtilde_v[b, j] = (1/H) * sum_h sum_{j'} Attn_h[j, j'] * m[b, j'],
+    where Attn_h is the row-softmax of sm_scale * q_{b,h,j} . k_{b,h,j'} (+ key_bias[b, j'])
+    over the keys j' <= j when causal, i.e. the attention matrix averaged over heads (eq. 3)
+    applied to the previous layer's vision score m (eq. 2 gives the hard labels at layer 0).
+
+    Q, K [B, H, S, hd]; m_keys [B, S]; key_bias [B, S] or None.
+    queries: None for all (b, j), else an int array [n, 2] of (b, j) rows to evaluate.
+    Returns Mtilde_v as [B, S] (queries None) or [n].
+    """
+    Q, K, m_keys = _f64(Q), _f64(K), _f64(m_keys)
+    B, H, S, _ = Q.shape
+    bias = np.zeros((B, S)) if key_bias is None else _f64(key_bias)
+
+    def one_query(b, j):
+        n = j + 1 if causal else S
+        logits = sm_scale * np.einsum('hd,hsd->hs', Q[b, :, j, :], K[b, :, :n, :]) + bias[b, None, :n]
+        logits = logits - logits.max(axis=1, keepdims=True)
+        w = np.exp(logits)
+        w = w / w.sum(axis=1, keepdims=True)
+        return float(np.mean(w @ m_keys[b, :n]))
+
+    if queries is None:
+        out = np.empty((B, S))
+        for b in range(B):
+            for h_block in range(0, S, 256):
+                # blocked evaluation of all queries of one sequence (same arithmetic as one_query)
+                j0, j1 = h_block, min(S, h_block + 256)
+                n = j1 if causal else S
+                logits = sm_scale * np.einsum('hqd,hsd->hqs', Q[b, :, j0:j1, :], K[b, :, :n, :])
+                logits = logits + bias[b, None, None, :n]
+                if causal:
+                    jj = np.arange(j0, j1)[:, None]
+                    kk = np.arange(n)[None, :]
+                    logits = np.where((kk <= jj)[None, :, :], logits, -np.inf)
+                logits = logits - logits.max(axis=2, keepdims=True)
+                w = np.exp(logits)
+                w = w / w.sum(axis=2, keepdims=True)
+                out[b, j0:j1] = np.mean(w @ m_keys[b, :n], axis=0)
+        return out
+    queries = np.asarray(queries)
+    return np.array([one_query(int(b), int(j)) for b, j in queries])
+
+
+def residual_score_update(M_tilde, M_prev, xattn_norm, x_norm):
+    """Residual-weighted score update, eq. (4):
+    M_next = (|x_attn| * Mtilde + |x| * M_prev) / (|x_attn| + |x|), per token and modality.
+    """
+    a = _f64(xattn_norm)
+    r = _f64(x_norm)
+    return (a * _f64(M_tilde) + r * _f64(M_prev)) / (a + r)
+
+
+# --------------------------------------------------------------------------------------------
+# Router: gate, softmax, top-k, bins (Sec. 3.1, Sec. 3.3)
+# --------------------------------------------------------------------------------------------
+
+def gate_logits(X, W):
+    """Gate logits z = W_gate x for every token (Sec. 3.1); X [T, d], W [E, d] -> z [T, E]."""
+    return _f64(X) @ _f64(W).T
+
+
+def softmax_gate(z):
+    """Gating scores g = softmax(z) over the routed experts (Sec. 3.1)."""
+    z = _f64(z)
+    e = np.exp(z - z.max(axis=1, keepdims=True))
+    return e / e.sum(axis=1, keepdims=True)
+
+
+def topk_route(z, g, k, renorm=False):
+    """Top-k expert choice (Sec. 3.1).
+
+    Order: descending logit; equal logits are ordered by ascending expert index (reading: the
+    paper does not fix a tie rule). Weights are the softmax scores of the chosen experts, or
+    those scores renormalised over the top-k when ``renorm``.
+    Returns (idx int32 [T, k], w float64 [T, k]).
+    """
+    z = _f64(z)
+    order = np.argsort(-z, axis=1, kind='stable')[:, :k]
+    w = np.take_along_axis(_f64(g), order, axis=1)
+    if renorm:
+        w = w / w.sum(axis=1, keepdims=True)
+    return order.astype(np.int32), w
+
+
+def bin_probs(g, expert_bin, n_bins):
+    """Per-bin routing probability p[j, k] = sum_{e in B_k} g[j, e] (the inner sum of eq. 12)."""
+    g = _f64(g)
+    expert_bin = np.asarray(expert_bin)
+    p = np.zeros((g.shape[0], n_bins))
+    for kb in range(n_bins):
+        p[:, kb] = g[:, expert_bin == kb].sum(axis=1)
+    return p
+
+
+# --------------------------------------------------------------------------------------------
+# Inter-bin mutual information (Sec. 3.4)
+# --------------------------------------------------------------------------------------------
+
+def sample_joint(M, p, N_B):
+    """Joint table of one sample, eqs. (12)-(14).
+
+    M [n, 2] soft scores, p [n, K] bin probabilities of the sample's tokens.
+      A[m]      = sum_j M[j, m]
+      Sbar[m,k] = sum_j M[j, m] p[j, k] / (N_B * A[m])           (12)
+      P[m,k]    = Sbar[m,k] / sum Sbar                            (13)
+      I         = sum_{m,k} P log(P / (P_m P_k)),  0 log 0 = 0    (14)
+    A modality with A[m] <= MASS_EPS is absent: its Sbar row is 0 (reading of 0/0).
+    Returns dict with A, N, Sbar, Z, P, Pm, Pk, I.
+    """
+    M, p = _f64(M), _f64(p)
+    K = p.shape[1]
+    A = M.sum(axis=0)
+    N = M.T @ p
+    Sbar = np.zeros((2, K))
+    for m in range(2):
+        if A[m] > MASS_EPS:
+            Sbar[m] = N[m] / (N_B * A[m])
+    Z = Sbar.sum()
+    P = Sbar / Z
+    Pm = P.sum(axis=1)
+    Pk = P.sum(axis=0)
+    I = 0.0
+    for m in range(2):
+        for kb in range(K):
+            if P[m, kb] > 0.0:
+                I += P[m, kb] * np.log(P[m, kb] / (Pm[m] * Pk[kb]))
+    return dict(A=A, N=N, Sbar=Sbar, Z=Z, P=P, Pm=Pm, Pk=Pk, I=I)
+
+
+def mi_loss(M, p, sample_offsets, N_B):
+    """Per-sample MI (eq. 14) and the MI loss of one layer, eq. (15): L = -(1/B) sum_i I_i.
+
+    M [T, 2], p [T, K], sample_offsets [B+1], N_B experts per bin.
+    Returns (mi [B], joint P [B, 2, K], loss, per-sample tables).
+    """
+    offs = np.asarray(sample_offsets)
+    B = len(offs) - 1
+    K = p.shape[1]
+    mis = np.zeros(B)
+    joint = np.zeros((B, 2, K))
+    tabs = []
+    for i in range(B):
+        s, e = int(offs[i]), int(offs[i + 1])
+        tab = sample_joint(M[s:e], p[s:e], N_B)
+        mis[i] = tab['I']
+        joint[i] = tab['P']
+        tabs.append(tab)
+    loss = -mis.sum() / B if B > 0 else 0.0
+    return mis, joint, loss, tabs
+
+
+def mi_grad_logits(M, g, expert_bin, sample_offsets, tabs, loss_scale, N_B):
+    """Gradient of loss_scale * L_MI with respect to the gate logits.
+
+    Derivation from eqs. (12)-(15), with the soft scores M (hence A) held constant
+    (stop-gradient; reading: the scores are guide signals, not functions of the gate):
+      dI/dSbar[m,k] = (log(P[m,k] / (P_m P_k)) - I) / Z
+      u[j,k]        = sum_m M[j,m] * dI/dSbar[m,k] / (N_B A[m])        (= dI/dg[j,e], e in B_k)
+      dI/dz[j,e]    = g[j,e] * (u[j, bin(e)] - sum_e' g[j,e'] u[j, bin(e')])   (softmax Jacobian)
+      dL/dz         = -(loss_scale / B) * dI/dz.
+    Absent modalities (A[m] <= MASS_EPS) contribute nothing.
+    """
+    M, g = _f64(M), _f64(g)
+    expert_bin = np.asarray(expert_bin)
+    offs = np.asarray(sample_offsets)
+    B = len(offs) - 1
+    dz = np.zeros_like(g)
+    for i in range(B):
+        s, e = int(offs[i]), int(offs[i + 1])
+        tab = tabs[i]
+        K = tab['P'].shape[1]
+        u_coef = np.zeros((2, K))
+        for m in range(2):
+            if tab['A'][m] > MASS_EPS:
+                with np.errstate(divide='ignore', invalid='ignore'):
+                    ratio = np.where(tab['P'][m] > 0, tab['P'][m] / (tab['Pm'][m] * tab['Pk']), 1.0)
+                dI_dS = (np.log(ratio) - tab['I']) / tab['Z']
+                u_coef[m] = dI_dS / (N_B * tab['A'][m])
+        u = M[s:e] @ u_coef                       # [n, K]
+        ue = u[:, expert_bin]                     # [n, E]
+        gi = g[s:e]
+        dI_dz = gi * (ue - np.sum(gi * ue, axis=1, keepdims=True))
+        dz[s:e] = -(loss_scale / B) * dI_dz
+    return dz
+
+
+def topk_weight_grad_logits(g, topk_idx, d_topk_w, renorm=False):
+    """Gradient reaching the gate logits from an upstream gradient of the top-k weights.
+
+    The weights are w_i = g[e_i] (or g[e_i] / sum_i' g[e_i'] when renormalised); the chain rule
+    through that renormalisation and through the softmax gives the returned dL/dz [T, E].
+    """
+    g = _f64(g)
+    T, E = g.shape
+    idx = np.asarray(topk_idx)
+    d = _f64(d_topk_w)
+    dg = np.zeros((T, E))
+    if renorm:
+        gsel = np.take_along_axis(g, idx, axis=1)
+        Gs = gsel.sum(axis=1, keepdims=True)
+        w = gsel / Gs
+        dsel = (d - np.sum(d * w, axis=1, keepdims=True)) / Gs
+    else:
+        dsel = d
+    rows = np.repeat(np.arange(T), idx.shape[1])
+    np.add.at(dg, (rows, idx.reshape(-1)), dsel.reshape(-1))
+    return g * (dg - np.sum(g * dg, axis=1, keepdims=True))
+
+
+# --------------------------------------------------------------------------------------------
+# Bin-grouped permutation and EP dispatch counts (Sec. 4.5, DeDup)
+# --------------------------------------------------------------------------------------------
+
+def expert_slots(expert_bin, n_bins):
+    """Position of every expert inside its bin (experts of a bin in ascending index order)."""
+    expert_bin = np.asarray(expert_bin)
+    slot = np.zeros(len(expert_bin), dtype=np.int64)
+    for kb in range(n_bins):
+        members = np.nonzero(expert_bin == kb)[0]
+        slot[members] = np.arange(len(members))
+    return slot
+
+
+def default_home(T, n_bins):
+    """Device a token lives on before dispatch (reading): a contiguous split over n_bins devices,
+    home(j) = floor(j * n_bins / T)."""
+    j = np.arange(T, dtype=np.int64)
+    return (j * n_bins) // max(T, 1)
+
+
+def bin_permute(topk_idx, expert_bin, n_bins, home=None, is_vision=None):
+    """De-duplicated bin dispatch (Sec. 4.5): one entry per unique (token, bin) pair.
+
+    A token is sent once to a bin even if several of its top-k experts live there; the entry
+    carries a bit mask of those experts (bit = the expert's slot inside the bin).
+    Order: bin ascending, token ascending inside a bin.
+    dispatch[h, k] counts unique pairs whose token lives on device h.
+    expert_counts[m, e] counts the tokens of hard modality m that chose expert e (eq. 10's C).
+    Returns dict(offsets [K+1], perm [P], mask [P], dispatch [K, K], expert_counts [2, E] or None).
+    """
+    idx = np.asarray(topk_idx, dtype=np.int64)
+    T, k = idx.shape
+    expert_bin = np.asarray(expert_bin, dtype=np.int64)
+    E = len(expert_bin)
+    K = n_bins
+    slot = expert_slots(expert_bin, K)
+    home = default_home(T, K) if home is None else np.asarray(home, dtype=np.int64)
+
+    sel_mask = np.zeros((T, K), dtype=np.uint64)          # bit mask of chosen experts per bin
+    bins = expert_bin[idx]                                # [T, k]
+    bits = np.left_shift(np.uint64(1), slot[idx].astype(np.uint64))
+    for c in range(k):
+        np.bitwise_or.at(sel_mask, (np.arange(T), bins[:, c]), bits[:, c])
+    present = sel_mask != 0                               # [T, K] unique pairs
+    counts = present.sum(axis=0)
+    offsets = np.zeros(K + 1, dtype=np.int64)
+    offsets[1:] = np.cumsum(counts)
+    # counting sort by bin, stable in token order
+    perm_parts, mask_parts = [], []
+    for kb in range(K):
+        toks = np.nonzero(present[:, kb])[0]
+        perm_parts.append(toks)
+        mask_parts.append(sel_mask[toks, kb])
+    perm = np.concatenate(perm_parts) if perm_parts else np.zeros(0, np.int64)
+    mask = np.concatenate(mask_parts) if mask_parts else np.zeros(0, np.uint64)
+    dispatch = np.zeros((K, K), dtype=np.int64)
+    jj, kk = np.nonzero(present)
+    np.add.at(dispatch, (home[jj], kk), 1)
+    ec = None
+    if is_vision is not None:
+        lab = np.where(np.asarray(is_vision) != 0, 0, 1)
+        ec = np.zeros((2, E), dtype=np.int64)
+        np.add.at(ec, (np.repeat(lab, k), idx.reshape(-1)), 1)
+    return dict(offsets=offsets, perm=perm, mask=mask, dispatch=dispatch, expert_counts=ec)
+
+
+# --------------------------------------------------------------------------------------------
+# Composite steps: one router layer forward and backward
+# --------------------------------------------------------------------------------------------
+
+def router_forward(X, W, M, expert_bin, n_bins, sample_offsets, k, renorm=False):
+    """Forward of one MoE router layer with the inter-bin MI regulariser (Secs. 3.1, 3.4).
+
+    X [T, d], W [E, d], M [T, 2] soft modality scores. Returns a dict with z, g, topk_idx,
+    topk_w, p, mi [B], joint [B, 2, K], loss and the per-sample tables (for the backward).
+    """
+    expert_bin = np.asarray(expert_bin)
+    N_B = len(expert_bin) // n_bins
+    z = gate_logits(X, W)
+    g = softmax_gate(z)
+    idx, w = topk_route(z, g, k, renorm)
+    p = bin_probs(g, expert_bin, n_bins)
+    mis, joint, loss, tabs = mi_loss(_f64(M), p, sample_offsets, N_B)
+    return dict(z=z, g=g, topk_idx=idx, topk_w=w, p=p, mi=mis, joint=joint, loss=loss, tabs=tabs)
+
+
+def router_backward(X, W, M, fwd, expert_bin, sample_offsets, loss_scale, d_topk_w=None,
+                    renorm=False):
+    """Backward of loss_scale * L_MI (+ an optional upstream gradient of the top-k weights).
+
+    dL/dz from mi_grad_logits (+ topk_weight_grad_logits), then dW = dz^T X and dX = dz W.
+    Returns (dz [T, E], dW [E, d], dX [T, d]).
+    """
+    expert_bin = np.asarray(expert_bin)
+    N_B = len(expert_bin) // fwd['p'].shape[1]
+    dz = mi_grad_logits(M, fwd['g'], expert_bin, sample_offsets, fwd['tabs'], loss_scale, N_B)
+    if d_topk_w is not None:
+        dz = dz + topk_weight_grad_logits(fwd['g'], fwd['topk_idx'], d_topk_w, renorm)
+    dW = dz.T @ _f64(X)
+    dX = dz @ _f64(W)
+    return dz, dW, dX
+
+
+def msi(expert_counts):
+    """Modality Specialization Index, eqs. (18)-(19), for one layer from counts C [2, E]
+    (row 0 vision, row 1 text). Returns a value in [0, 1]."""
+    C = _f64(expert_counts)
+    share = C / C.sum(axis=1, keepdims=True)            # C_{m,e} / sum_e' C_{m,e'}
+    Ct = share / share.sum(axis=0, keepdims=True)       # eq. (18)
+    return float(np.mean(2.0 * np.abs(Ct[1] - 0.5)))    # eq. (19), text row
