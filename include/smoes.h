@@ -1,0 +1,190 @@
+/*
+ * smoes.h -- C ABI of the GB300 (sm_103a) SMoES router hot path.
+ *
+ * SMoES ("Soft Modality-Guided Expert Specialization in MoE-VLMs") regularises an MoE router
+ * so that groups of experts ("bins") specialise by modality. Per MoE layer the hot path is:
+ *   soft modality score (Sec. 3.2: Gaussian statistics, eqs. (8)-(9), or attention mass,
+ *   eqs. (2)-(4)) -> gate logits z = W x, softmax, top-k (Sec. 3.1) -> expert-to-bin sums
+ *   -> per-sample inter-bin mutual information and the MI loss (Sec. 3.4, eqs. (12)-(15))
+ *   -> gradient of the MI loss to W and x -> bin-grouped token permutation with
+ *   de-duplicated expert-parallel dispatch counts (Sec. 4.5).
+ *
+ * Conventions shared by every call
+ *   - Arrays are dense, row-major, device pointers, 16-byte aligned; the caller owns every
+ *     buffer, including the workspace. The library never allocates device memory.
+ *   - X is [T, d] (tokens x hidden), W is [E, d] (the torch Linear layout of W_gate).
+ *   - Modality index 0 = vision, 1 = text. M is [T, 2] float32, rows sum to 1.
+ *   - Sample i (the paper's index i) is the contiguous token range
+ *     [sample_offsets[i], sample_offsets[i+1]).
+ *   - All work is enqueued asynchronously on the given stream. Argument errors are found on the
+ *     host before any launch and leave every output untouched. Errors found while kernels run
+ *     (non-finite values, non-positive variances, invalid indices, a bounded device wait that
+ *     ran out) set a status word inside the workspace; read it with smoes_read_device_status.
+ *   - Calls that share one workspace must be ordered on the GPU (same stream, or synchronised).
+ */
+#ifndef SMOES_H
+#define SMOES_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SMOES_OK = 0,
+  SMOES_ERR_INVALID_ARG = -1,     /* bad size, pointer, map or offsets; nothing launched      */
+  SMOES_ERR_UNSUPPORTED = -2,     /* valid but outside what this build supports              */
+  SMOES_ERR_ALIGNMENT = -3,       /* a pointer is not 16-byte aligned                        */
+  SMOES_ERR_WORKSPACE = -4,       /* workspace missing or smaller than smoes_workspace_bytes */
+  SMOES_ERR_CUDA = -5,            /* a CUDA runtime/driver call or a launch failed           */
+  SMOES_ERR_DEVICE_TIMEOUT = -6,  /* (device status) a bounded wait inside a kernel expired  */
+  SMOES_ERR_DATA = -7             /* (device status) non-finite or out-of-range input data   */
+} smoes_status;
+
+typedef enum { SMOES_F32 = 0, SMOES_BF16 = 1 } smoes_dtype;
+
+typedef enum {
+  SMOES_SCORE_PROVIDED = 0,       /* M is given by the caller                       */
+  SMOES_SCORE_GAUSS = 1,          /* Gaussian-statistics score, eqs. (8)-(9)        */
+  SMOES_SCORE_ATTN = 2            /* attention-accumulated score, eqs. (2)-(4)      */
+} smoes_score_mode;
+
+typedef struct smoes_plan_s* smoes_plan;
+
+/* Shape and routing metadata of one router layer (Secs. 3.1, 3.3).
+ *   T >= 0 tokens; d hidden size (d % 8 == 0, d >= 8); E routed experts (1..256);
+ *   k top-k (1..16, k <= E); n_bins bins (1..32, E % n_bins == 0, E / n_bins <= 32);
+ *   n_samples >= 1 when T > 0 (0 when T == 0).
+ *   sample_offsets_host [n_samples+1]: 0 = o_0 < o_1 < ... < o_B = T (no empty sample).
+ *   expert_bin_host [E]: bin of each expert, each bin holding exactly E / n_bins experts.
+ *   renorm_topk: 0 -> top-k weights are the softmax scores; 1 -> renormalised over the top-k.
+ *   attn_max_heads: largest head count passed to smoes_modality_score(SMOES_SCORE_ATTN)
+ *   (sizes the per-head partial sums in the workspace); 0 if the attention score is not used.
+ * Both host arrays are copied; the caller may free them after smoes_plan_create returns. */
+typedef struct {
+  int T, d, E, k, n_bins, n_samples;
+  smoes_dtype dtype;                   /* element type of X, W and dX                          */
+  const int32_t* sample_offsets_host;
+  const int32_t* expert_bin_host;
+  int renorm_topk;
+  int attn_max_heads;
+} smoes_router_desc;
+
+/* Gaussian-statistics score inputs, eqs. (8)-(9).
+ *   X [T, d] (plan dtype); mu, var [2, d] float32 (row 0 vision, row 1 text), var > 0;
+ *   tau > 0 the temperature, or tau <= 0 for the paper's default 0.5 * d (Sec. 4.1). */
+typedef struct {
+  const void* X;
+  const float* mu;
+  const float* var;
+  float tau;
+} smoes_gauss_args;
+
+/* Attention-accumulated score inputs, eqs. (2)-(4).
+ *   Q, K [B, H, S, hd] bf16 with B * S == T (token b*S + j is query j of sequence b);
+ *   hd % 16 == 0, hd <= 256.
+ *   Exactly one of is_vision ([T] uint8, the hard labels of eq. (2)) or m_prev ([T] float32,
+ *   the previous layer's vision score) gives the score carried by every key.
+ *   key_bias [T] float32 or NULL: added to the logit of key j of its sequence.
+ *   sm_scale: logit scale (1/sqrt(hd) for standard attention). causal: 1 = keys j' <= j only.
+ *   xattn_norm, x_norm [T] float32 or NULL: when both are given, eq. (4) blends the aggregated
+ *   score with the carried one, weighted by |x_attn| and |x|.                               */
+typedef struct {
+  const void* Q;
+  const void* K;
+  int B, H, S, hd;
+  const uint8_t* is_vision;
+  const float* m_prev;
+  const float* key_bias;
+  float sm_scale;
+  int causal;
+  const float* xattn_norm;
+  const float* x_norm;
+} smoes_attn_args;
+
+typedef struct {
+  smoes_gauss_args gauss;
+  smoes_attn_args attn;
+} smoes_score_args;
+
+/* Validates the descriptor and builds the host-side plan (no device memory is touched).
+ * Returns SMOES_ERR_INVALID_ARG / SMOES_ERR_UNSUPPORTED on bad or unsupported shapes. */
+smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out);
+void smoes_plan_destroy(smoes_plan plan);
+
+/* Bytes of device workspace the plan needs (metadata, forward-to-backward state, partial sums,
+ * status word). The workspace is caller-owned and 256-byte aligned. */
+size_t smoes_workspace_bytes(smoes_plan plan);
+
+/* Writes the plan's metadata into the workspace and clears its counters and status word.
+ * Call once after allocating the workspace (and again after any device-side error), on the
+ * stream that later calls use. */
+smoes_status smoes_workspace_init(smoes_plan plan, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+const char* smoes_status_string(smoes_status status);
+
+/* Synchronises `stream`, reads the workspace status word and returns SMOES_OK,
+ * SMOES_ERR_DATA or SMOES_ERR_DEVICE_TIMEOUT. *n_absent_modality (optional) receives how many
+ * (sample, modality) pairs had zero soft mass in the last forward (eq. (12) read as 0). */
+smoes_status smoes_read_device_status(smoes_plan plan, const void* ws, cudaStream_t stream,
+                                      int32_t* n_absent_modality);
+
+/* (1) Soft modality score (Sec. 3.2).
+ *   mode SMOES_SCORE_GAUSS: M[j] = softmax_m(LL[j, m] / tau) with LL of eq. (8).
+ *   mode SMOES_SCORE_ATTN:  M[j, 0] = (1/H) sum_h sum_j' softmax_j'(s q.k_j' + bias_j') m_j'
+ *                           (eq. (3), optionally followed by eq. (4)); M[j, 1] = 1 - M[j, 0].
+ *   M: [T, 2] float32 output. ws is needed by SMOES_SCORE_ATTN (head partial sums). */
+smoes_status smoes_modality_score(smoes_plan plan, smoes_score_mode mode,
+                                  const smoes_score_args* args, float* M,
+                                  void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* (2) Router forward with the MI regulariser (Secs. 3.1, 3.3, 3.4).
+ *   X [T, d], W [E, d] (plan dtype). Scores: M_in [T, 2] (SMOES_SCORE_PROVIDED, gauss == NULL),
+ *   or gauss != NULL (fused Gaussian score; gauss->X is ignored, X is used) and the scores are
+ *   written to M_out [T, 2] (required then).
+ *   Outputs: topk_idx [T, k] int32 (descending logit, equal logits -> lower expert index),
+ *   topk_w [T, k] float32, bin_prob [T, n_bins] float32 (optional, NULL to skip),
+ *   joint [B, 2, n_bins] float32 P_i(m, B_k) of eq. (13) (optional), mi [B] float32 I_i of
+ *   eq. (14), loss [1] float32 = -(1/B) sum_i I_i (eq. (15), one layer).
+ *   ws keeps the softmax scores and per-sample tables that smoes_router_bwd reads. */
+smoes_status smoes_router_fwd(smoes_plan plan, const void* X, const void* W, const float* M_in,
+                              const smoes_gauss_args* gauss, float* M_out,
+                              int32_t* topk_idx, float* topk_w, float* bin_prob,
+                              float* joint, float* mi, float* loss,
+                              void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* (3) Backward of loss_scale * L_MI (plus, optionally, an upstream gradient of topk_w).
+ *   The soft scores are constants (no gradient flows into M). X, W, M and topk_idx must be the
+ *   tensors of the preceding smoes_router_fwd on the same ws.
+ *   dW [E, d] float32: written, or accumulated into when accumulate_dW != 0.
+ *   dX [T, d] (plan dtype) or NULL; dlogits [T, E] float32 or NULL.
+ *   d_topk_w [T, k] float32 or NULL. */
+smoes_status smoes_router_bwd(smoes_plan plan, const void* X, const void* W, const float* M,
+                              const int32_t* topk_idx, const float* d_topk_w, float loss_scale,
+                              float* dW, int accumulate_dW, void* dX, float* dlogits,
+                              void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* (4) Bin-grouped permutation with de-duplicated dispatch (Sec. 4.5, "DeDup").
+ *   One entry per unique (token, bin) pair, ordered by bin ascending then token ascending.
+ *   topk_idx [T, k] int32 in [0, E). home [T] int32 in [0, n_bins) or NULL for the contiguous
+ *   split home(j) = floor(j * n_bins / T). is_vision [T] uint8 (required if expert_counts).
+ *   Outputs: bin_offsets [n_bins+1] int32; perm_token and perm_mask with capacity
+ *   T * min(k, n_bins) (bit s of perm_mask = the expert in slot s of the bin, slots ordering a
+ *   bin's experts by index); dispatch [n_bins, n_bins] int32, dispatch[h][b] = pairs whose
+ *   token lives on device h and goes to bin b; expert_counts [2, E] int32 (optional) = tokens
+ *   of each hard modality that chose each expert (the count C_{m,e} of eq. (10)). */
+smoes_status smoes_bin_permute(smoes_plan plan, const int32_t* topk_idx, const int32_t* home,
+                               const uint8_t* is_vision, int32_t* bin_offsets,
+                               int32_t* perm_token, uint32_t* perm_mask, int32_t* dispatch,
+                               int32_t* expert_counts, void* ws, size_t ws_bytes,
+                               cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SMOES_H */

@@ -1,0 +1,533 @@
+// router_bwd.cu -- backward of loss_scale * L_MI (eq. 15) on sm_103a.
+//
+// With the soft scores held constant, the gradient reaching the gate logits is
+//   dz_je = scale * g_je * (u_j,b(e) - sum_e' g_je' u_j,b(e'))           (scale = -loss_scale/B)
+//   u_jk  = h_k + (M_jv - 1/2) a_k + (M_jt - 1/2) b_k
+// with the per-sample coefficients (a, b, h) written by the forward. Optionally an upstream
+// gradient of the top-k weights is pushed through the (renormalised) softmax as well.
+// Then dW = dz^T X and dX = dz W.
+//
+// tcgen05 path (bf16): CTA (token group g, d-slice s). Per 64-token tile, four "dz" warps build
+// dz in shared memory as a bf16 hi/lo pair (dz = hi + lo to ~2^-17 relative), and one thread
+// issues, per 128-column d-block of the slice,
+//   dW^T[d-block] += X^T(tile) . dz        (M = 128 d, N = E_pad, K = 64 tokens)  -> TMEM, kept
+//   dX^T[d-block]  = W^T(d-block) . dz^T   (M = 128 d, N = 64 tokens, K = E_pad)  -> TMEM, drained
+// X tiles arrive by TMA; the W slice stays resident in shared memory; dX leaves by TMA store.
+// The per-group dW^T slice is written once at the end and summed over groups in fixed order.
+#include <cuda_bf16.h>
+
+#include "ptx.cuh"
+#include "smoes_internal.cuh"
+
+namespace smoes {
+namespace {
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat16 a = __float2bfloat16_rn(lo), b = __float2bfloat16_rn(hi);
+  return static_cast<uint32_t>(__bfloat16_as_ushort(a)) |
+         (static_cast<uint32_t>(__bfloat16_as_ushort(b)) << 16);
+}
+
+// Upstream top-k weight gradient of one token, folded into per-expert terms:
+//   dt[e] = sum over top-k slots i with idx_i == e of dtil_i, and gdt = sum_i g_{idx_i} dtil_i,
+// where dtil_i = d_i (raw weights) or (d_i - sum_i' d_i' w_i') / G (renormalised, G = sum g_sel).
+struct Upstream {
+  int idx[kMaxTopK];
+  float dtil[kMaxTopK];
+  float gdt;
+};
+
+__device__ __forceinline__ void load_upstream(const BwdParams& p, int j, Upstream& u) {
+  const int k = p.dm.k;
+  float gsel[kMaxTopK], d[kMaxTopK];
+  float G = 0.f, dw = 0.f;
+  const float* g = p.ws.gsave + static_cast<size_t>(j) * p.dm.E;
+#pragma unroll
+  for (int i = 0; i < kMaxTopK; ++i) {
+    u.idx[i] = -1;
+    u.dtil[i] = 0.f;
+    gsel[i] = 0.f;
+    d[i] = 0.f;
+    if (i < k) {
+      u.idx[i] = p.topk_idx[static_cast<size_t>(j) * k + i];
+      d[i] = p.d_topk_w[static_cast<size_t>(j) * k + i];
+      const int e = u.idx[i];
+      gsel[i] = (e >= 0 && e < p.dm.E) ? g[e] : 0.f;
+      G += gsel[i];
+    }
+  }
+  if (p.dm.renorm) {
+#pragma unroll
+    for (int i = 0; i < kMaxTopK; ++i)
+      if (i < k) dw += d[i] * gsel[i] / G;
+  }
+  float gdt = 0.f;
+#pragma unroll
+  for (int i = 0; i < kMaxTopK; ++i) {
+    if (i < k) {
+      u.dtil[i] = p.dm.renorm ? (d[i] - dw) / G : d[i];
+      gdt += gsel[i] * u.dtil[i];
+    }
+  }
+  u.gdt = gdt;
+}
+
+__device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
+  float r = 0.f;
+#pragma unroll
+  for (int i = 0; i < kMaxTopK; ++i)
+    if (i < k && u.idx[i] == e) r += u.dtil[i];
+  return r;
+}
+
+// ------------------------------------------------------------------ tcgen05 backward (bf16)
+
+struct BwdLayout {
+  uint32_t wsl, dz, xst, stg, ubar, us, bars, total;
+};
+
+__host__ __device__ inline BwdLayout bwd_layout(int E_pad, int n_xst, int K) {
+  BwdLayout L;
+  uint32_t o = 0;
+  L.wsl = o;  o += 65536u;                                     // W slice (ds * E_pad * 2 B)
+  L.dz = o;   o += 2u * 2u * static_cast<uint32_t>(E_pad) * 128u; // 2 buffers x (hi, lo)
+  L.xst = o;  o += static_cast<uint32_t>(n_xst) * 16384u;     // X stages [2 atoms][64][128 B]
+  L.stg = o;  o += 2u * 16384u;                                // dX staging [64][128] bf16 x2
+  L.ubar = o; o += 2u * 2u * 64u * 4u;                         // [2 buf][2 half][64]
+  L.us = o;   o += static_cast<uint32_t>(K) * 128u * 4u;       // [K][128]
+  L.bars = o; o += 8u * (2u * n_xst + 18u) + 16u;
+  L.total = o + 1024u;
+  return L;
+}
+
+__global__ void __launch_bounds__(320, 1)
+k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
+                const __grid_constant__ CUtensorMap tmDX, const BwdParams p, const int E_pad,
+                const int n_xst) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const Dims& dm = p.dm;
+  const BwdLayout L = bwd_layout(E_pad, n_xst, dm.K);
+  uint8_t* wsl = base + L.wsl;
+  uint8_t* dzb = base + L.dz;               // buffer zb: hi at zb*2*E_pad*128, lo right after
+  uint8_t* xst = base + L.xst;
+  uint8_t* stg = base + L.stg;
+  float* ubar = reinterpret_cast<float*>(base + L.ubar);
+  float* us = reinterpret_cast<float*>(base + L.us);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
+  uint64_t* xfull = bars;
+  uint64_t* xempty = bars + n_xst;
+  uint64_t* dz_full = bars + 2 * n_xst;       // [2]
+  uint64_t* dz_empty = dz_full + 2;           // [2]
+  uint64_t* dx_full = dz_full + 4;            // [2]
+  uint64_t* dx_empty = dz_full + 6;           // [2]
+  uint64_t* wfull = dz_full + 8;
+  uint64_t* dw_full = dz_full + 9;
+  uint64_t* drain = dz_full + 10;
+  uint64_t* ub_bar = dz_full + 11;            // [2] dz warps exchange half sums
+  uint64_t* stg_free = dz_full + 13;          // [2] staging buffer may be rewritten
+  uint64_t* stg_full = dz_full + 15;          // [2] staging buffer written
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dz_full + 18);
+  int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int S = p.slices, G = p.groups;
+  const int sl = blockIdx.x % S, grp = blockIdx.x / S;
+  const int d0 = sl * p.slice_width;
+  const int nb = min(p.slice_width, round_up(dm.d - d0, kBwdBD)) / kBwdBD;   // d-blocks here
+  const bool want_dx = p.dX != nullptr;
+  const uint32_t dz_buf_bytes = 2u * static_cast<uint32_t>(E_pad) * 128u;   // hi + lo
+  const uint32_t dz_half = static_cast<uint32_t>(E_pad) * 128u;             // one of hi / lo
+  WaitCtx wc{abort_flag, p.ws.status, p.limit_ns};
+
+  if (threadIdx.x == 0) {
+    *abort_flag = 0;
+    for (int i = 0; i < n_xst; ++i) {
+      mbar_init(xfull + i, 1);
+      mbar_init(xempty + i, 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(dz_full + i, 128);
+      mbar_init(dz_empty + i, 1);
+      mbar_init(dx_full + i, 1);
+      mbar_init(dx_empty + i, 128);
+      mbar_init(ub_bar + i, 128);
+      mbar_init(stg_free + i, 1);
+      mbar_init(stg_full + i, 128);
+    }
+    mbar_init(wfull, 1);
+    mbar_init(dw_full, 1);
+    mbar_init(drain, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tmX);
+    tma_prefetch_desc(&tmW);
+    tma_prefetch_desc(&tmDX);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t tm_dx = tmem + 256u;          // two 64-column dX^T buffers after the dW^T blocks
+
+  if (warp == 0) {
+    // -------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      bool ok = true;
+      mbar_arrive_expect_tx(wfull, static_cast<uint32_t>(nb) * 2u * dz_half);
+      for (int a = 0; a < 2 * nb; ++a)        // W slice: atom a = columns d0 + 64a .. +64
+        tma_load_2d(wsl + a * dz_half, &tmW, wfull, d0 + 64 * a, 0);
+      int st = 0;
+      uint32_t ph = 0;
+      long issued = 0;
+      for (int t = grp; t < p.n_tiles && ok; t += G) {
+        for (int b = 0; b < nb; ++b) {
+          if (!mbar_wait(xempty + st, ph ^ 1u, wc)) { ok = false; break; }
+          uint8_t* xs = xst + st * 16384;
+          mbar_arrive_expect_tx(xfull + st, 16384u);
+          tma_load_2d(xs, &tmX, xfull + st, d0 + b * kBwdBD, t * kBwdBT);
+          tma_load_2d(xs + 8192, &tmX, xfull + st, d0 + b * kBwdBD + 64, t * kBwdBT);
+          ++issued;
+          if (++st == n_xst) { st = 0; ph ^= 1u; }
+        }
+      }
+      WaitCtx wd = wc;
+      int dummy = 0;
+      wd.abort_flag = &dummy;
+      mbar_wait(wfull, 0, wd);                // the W slice copy must land before exit
+      if (!ok) {
+        for (long q = (issued > n_xst ? issued - n_xst : 0); q < issued; ++q)
+          mbar_wait(xfull + (q % n_xst), static_cast<uint32_t>((q / n_xst) & 1), wd);
+      }
+    }
+  } else if (warp == 1) {
+    // -------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t id_dw = idesc_bf16(128, E_pad, true, true);
+      const uint32_t id_dx = idesc_bf16(128, kBwdBT, true, false);
+      bool ok = mbar_wait(wfull, 0, wc);
+      tc_fence_after();
+      int st = 0, xb = 0;
+      uint32_t ph = 0, xph = 0;
+      int lt = 0;
+      for (int t = grp; t < p.n_tiles && ok; t += G, ++lt) {
+        const int zb = lt & 1;
+        const uint32_t zuse = static_cast<uint32_t>(lt >> 1);
+        if (!mbar_wait(dz_full + zb, zuse & 1u, wc)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t hi = smem_u32(dzb + zb * dz_buf_bytes);
+        const uint32_t lo = hi + dz_half;
+        for (int b = 0; b < nb; ++b) {
+          if (!mbar_wait(xfull + st, ph, wc)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t xs = smem_u32(xst + st * 16384);
+          const uint32_t dwc = tmem + static_cast<uint32_t>(b * E_pad);
+#pragma unroll
+          for (int ks = 0; ks < kBwdBT / 16; ++ks) {     // K = 16 tokens per instruction
+            const uint64_t da = sdesc_sw128(xs + ks * 2048, 8192, 1024);
+            const uint64_t dh = sdesc_sw128(hi + ks * 2048, 8192, 1024);
+            const uint64_t dl = sdesc_sw128(lo + ks * 2048, 8192, 1024);
+            umma_bf16(dwc, da, dh, id_dw, (lt > 0 || ks > 0) ? 1u : 0u);
+            umma_bf16(dwc, da, dl, id_dw, 1u);
+          }
+          if (want_dx) {
+            if (!mbar_wait(dx_empty + xb, xph ^ 1u, wc)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t dxc = tm_dx + static_cast<uint32_t>(xb * kBwdBT);
+            const uint32_t wa = smem_u32(wsl + 2 * b * dz_half);
+            for (int ke = 0; ke < E_pad / 16; ++ke) {    // K = 16 experts per instruction
+              const uint64_t da = sdesc_sw128(wa + ke * 2048, dz_half, 1024);
+              const uint32_t boff = (ke >> 2) * 8192 + (ke & 3) * 32;
+              const uint64_t dh = sdesc_sw128(hi + boff, 16, 1024);
+              const uint64_t dl = sdesc_sw128(lo + boff, 16, 1024);
+              umma_bf16(dxc, da, dh, id_dx, ke > 0 ? 1u : 0u);
+              umma_bf16(dxc, da, dl, id_dx, 1u);
+            }
+            umma_commit(dx_full + xb);
+            if (++xb == 2) { xb = 0; xph ^= 1u; }
+          }
+          umma_commit(xempty + st);
+          if (++st == n_xst) { st = 0; ph ^= 1u; }
+        }
+        if (!ok) break;
+        umma_commit(dz_empty + zb);
+      }
+      if (ok) umma_commit(dw_full);
+      umma_commit(drain);
+      WaitCtx wd = wc;
+      int dummy = 0;
+      wd.abort_flag = &dummy;
+      mbar_wait(drain, 0, wd);
+    }
+  } else if (warp < 6) {
+    // -------------------------------------------------------------- dX epilogue + dW drain
+    const int lg = warp & 3;
+    const int etid = threadIdx.x - 64;                 // 0..127
+    const bool issuer = (etid == 0);
+    int xb = 0;
+    uint32_t xph = 0;
+    int it = 0;
+    bool ok = true;
+    if (want_dx) {
+      for (int t = grp; t < p.n_tiles && ok; t += G) {
+        for (int b = 0; b < nb; ++b, ++it) {
+          if (!mbar_wait(dx_full + xb, xph, wc)) { ok = false; break; }
+          tc_fence_after();
+          const int sb = it & 1;
+          const uint32_t suse = static_cast<uint32_t>(it >> 1);
+          if (issuer) {                                // staging[sb] free again
+            tma_store_wait_read<1>();
+            mbar_arrive(stg_free + sb);
+          }
+          if (!mbar_wait(stg_free + sb, suse & 1u, wc)) { ok = false; break; }
+          __nv_bfloat16* sg = reinterpret_cast<__nv_bfloat16*>(stg + sb * 16384);
+          const uint32_t ta = tm_dx + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(xb * kBwdBT);
+          const int drow = lg * 32 + lane;
+#pragma unroll
+          for (int c = 0; c < kBwdBT / 16; ++c) {
+            float v[16];
+            tmem_ld16(ta + 16u * c, v);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) sg[(c * 16 + q) * kBwdBD + drow] = __float2bfloat16_rn(v[q]);
+          }
+          tc_fence_before();
+          mbar_arrive(dx_empty + xb);
+          if (++xb == 2) { xb = 0; xph ^= 1u; }
+          fence_proxy_async_smem();
+          mbar_arrive(stg_full + sb);
+          if (issuer) {
+            if (!mbar_wait(stg_full + sb, suse & 1u, wc)) { ok = false; break; }
+            tma_store_2d(&tmDX, sg, d0 + b * kBwdBD, t * kBwdBT);
+            tma_store_commit();
+          }
+        }
+      }
+      if (issuer) tma_store_wait_all<0>();
+    }
+    // partial dW^T of this group: lanes = d rows, columns = experts
+    if (ok && mbar_wait(dw_full, 0, wc)) {
+      tc_fence_after();
+      for (int b = 0; b < nb; ++b) {
+        const int drow = d0 + b * kBwdBD + lg * 32 + lane;
+        const uint32_t ta = tmem + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(b * E_pad);
+        for (int c = 0; c < E_pad / 16; ++c) {
+          float v[16];
+          tmem_ld16(ta + 16u * c, v);
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            const int e = c * 16 + q;
+            if (e < dm.E && drow < dm.d)
+              p.ws.dw_part[(static_cast<size_t>(grp) * dm.E + e) * dm.d + drow] = v[q];
+          }
+        }
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- dz producers (4 warps)
+    const int w4 = warp - 6;
+    const int r = (w4 & 1) * 32 + lane;                // token row in the tile
+    const int h = w4 >> 1;                             // expert half
+    const int dtid = threadIdx.x - 192;                // 0..127
+    const int Eh = E_pad / 2;
+    const int K = dm.K, E = dm.E, k = dm.k;
+    const float* gs = p.ws.gsave;
+    int lt = 0;
+    for (int t = grp; t < p.n_tiles; t += G, ++lt) {
+      const int zb = lt & 1;
+      const uint32_t zuse = static_cast<uint32_t>(lt >> 1);
+      if (!mbar_wait(dz_empty + zb, (zuse & 1u) ^ 1u, wc)) break;
+      const int j = t * kBwdBT + r;
+      const bool valid = j < dm.T;
+      float dv = 0.f, dt = 0.f;
+      if (valid) {
+        const int s = p.ws.token_sample[j];
+        const float2 m = *reinterpret_cast<const float2*>(p.M + 2 * static_cast<size_t>(j));
+        dv = m.x - 0.5f;
+        dt = m.y - 0.5f;
+        const float* tb = p.ws.tabs + static_cast<size_t>(s) * 3 * K;
+        for (int kb = 0; kb < K; ++kb)
+          us[kb * 128 + dtid] = __ldcg(tb + 2 * K + kb) + dv * __ldcg(tb + kb) + dt * __ldcg(tb + K + kb);
+      }
+      Upstream up;
+      const bool has_up = valid && p.d_topk_w != nullptr;
+      if (has_up) load_upstream(p, j, up);
+      // partial  sum_e g_e u_b(e)  over this thread's experts
+      float part = 0.f;
+      const int e0 = h * Eh;
+      for (int e = e0; e < e0 + Eh; ++e) {
+        if (valid && e < E) part += __ldcg(gs + static_cast<size_t>(j) * E + e) * us[p.ws.expert_bin[e] * 128 + dtid];
+      }
+      ubar[(zb * 2 + h) * 64 + r] = part;
+      mbar_arrive(ub_bar + zb);
+      if (!mbar_wait(ub_bar + zb, zuse & 1u, wc)) break;
+      const float ub = ubar[(zb * 2 + 0) * 64 + r] + ubar[(zb * 2 + 1) * 64 + r];
+      uint8_t* hib = dzb + zb * dz_buf_bytes;
+      uint8_t* lob = hib + dz_half;
+      for (int c = 0; c < Eh / 8; ++c) {
+        const int eb = e0 + c * 8;
+        float dz[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const int e = eb + q;
+          float v = 0.f;
+          if (valid && e < E) {
+            const float g = __ldcg(gs + static_cast<size_t>(j) * E + e);
+            v = p.scale * g * (us[p.ws.expert_bin[e] * 128 + dtid] - ub);
+            if (has_up) v += g * (upstream_at(up, k, e) - up.gdt);
+          }
+          dz[q] = v;
+        }
+        if (valid && p.dlogits) {
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            if (eb + q < E) p.dlogits[static_cast<size_t>(j) * E + eb + q] = dz[q];
+        }
+        uint32_t hw[4], lw[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const __nv_bfloat16 h0 = __float2bfloat16_rn(dz[2 * q]), h1 = __float2bfloat16_rn(dz[2 * q + 1]);
+          hw[q] = static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
+          lw[q] = pack_bf16x2(dz[2 * q] - __bfloat162float(h0), dz[2 * q + 1] - __bfloat162float(h1));
+        }
+        const uint32_t off = (eb >> 6) * 8192u + sw128_offset(static_cast<uint32_t>(r), static_cast<uint32_t>(eb & 63));
+        *reinterpret_cast<uint4*>(hib + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *reinterpret_cast<uint4*>(lob + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(dz_full + zb);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// ------------------------------------------------------------------ FFMA backward (fp32)
+// One block per 64-token tile, all of d. dz for the tile is built in shared memory
+// (4 threads per token); then each thread owns one column per 256-column chunk, produces dX
+// for the tile and accumulates the tile's partial dW^T column in registers.
+constexpr int kF32MaxE = 64;
+
+__global__ void __launch_bounds__(256)
+k_router_bwd_f32(const BwdParams p) {
+  extern __shared__ float bs[];
+  const Dims& dm = p.dm;
+  const int E = dm.E, K = dm.K, k = dm.k;
+  float* dzs = bs;                                   // [64][E+1]
+  const int t = threadIdx.x;
+  const int tile = blockIdx.x;
+  {
+    const int r = t >> 2, qd = t & 3;
+    const int j = tile * 64 + r;
+    const bool valid = j < dm.T;
+    float dv = 0.f, dt = 0.f;
+    const float* tb = nullptr;
+    if (valid) {
+      const int s = p.ws.token_sample[j];
+      dv = p.M[2 * static_cast<size_t>(j)] - 0.5f;
+      dt = p.M[2 * static_cast<size_t>(j) + 1] - 0.5f;
+      tb = p.ws.tabs + static_cast<size_t>(s) * 3 * K;
+    }
+    Upstream up;
+    const bool has_up = valid && p.d_topk_w != nullptr;
+    if (has_up) load_upstream(p, j, up);
+    const float* g = p.ws.gsave + static_cast<size_t>(valid ? j : 0) * E;
+    float part = 0.f;
+    for (int e = qd; e < E; e += 4) {
+      if (valid) {
+        const int b = p.ws.expert_bin[e];
+        part += g[e] * (tb[2 * K + b] + dv * tb[b] + dt * tb[K + b]);
+      }
+    }
+    part += __shfl_xor_sync(0xffffffffu, part, 1);
+    part += __shfl_xor_sync(0xffffffffu, part, 2);
+    for (int e = qd; e < E; e += 4) {
+      float v = 0.f;
+      if (valid) {
+        const int b = p.ws.expert_bin[e];
+        const float u = tb[2 * K + b] + dv * tb[b] + dt * tb[K + b];
+        v = p.scale * g[e] * (u - part);
+        if (has_up) v += g[e] * (upstream_at(up, k, e) - up.gdt);
+        if (p.dlogits) p.dlogits[static_cast<size_t>(j) * E + e] = v;
+      }
+      dzs[r * (E + 1) + e] = v;
+    }
+  }
+  __syncthreads();
+  const float* X = static_cast<const float*>(p.X);
+  const float* W = static_cast<const float*>(p.W);
+  float* dX = static_cast<float*>(p.dX);
+  const int rows = min(64, dm.T - tile * 64);
+  for (int c0 = 0; c0 < dm.d; c0 += 256) {
+    const int c = c0 + t;
+    if (c >= dm.d) break;
+    float wc[kF32MaxE], acc[kF32MaxE];
+#pragma unroll
+    for (int e = 0; e < kF32MaxE; ++e) {
+      wc[e] = (e < E) ? W[static_cast<size_t>(e) * dm.d + c] : 0.f;
+      acc[e] = 0.f;
+    }
+    for (int r = 0; r < rows; ++r) {
+      const size_t j = static_cast<size_t>(tile) * 64 + r;
+      const float x = X[j * dm.d + c];
+      float dx = 0.f;
+#pragma unroll
+      for (int e = 0; e < kF32MaxE; ++e) {
+        if (e < E) {
+          const float z = dzs[r * (E + 1) + e];
+          dx = fmaf(z, wc[e], dx);
+          acc[e] = fmaf(z, x, acc[e]);
+        }
+      }
+      if (dX) dX[j * dm.d + c] = dx;
+    }
+#pragma unroll
+    for (int e = 0; e < kF32MaxE; ++e)
+      if (e < E) p.ws.dw_part[(static_cast<size_t>(tile) * E + e) * dm.d + c] = acc[e];
+  }
+}
+
+// dW[e][c] = (accumulate ? dW[e][c] : 0) + sum_{g=0}^{G-1} part[g][e][c], in that order.
+__global__ void k_dw_reduce(const BwdParams p) {
+  const size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
+  const size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  float acc = p.accumulate ? p.dW[i] : 0.f;
+  for (int g = 0; g < p.groups; ++g) acc += __ldcg(p.ws.dw_part + static_cast<size_t>(g) * n + i);
+  p.dW[i] = acc;
+}
+
+}  // namespace
+
+cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, const CUtensorMap& tmW,
+                                   const CUtensorMap& tmDX, cudaStream_t s) {
+  const int E_pad = round_up(p.dm.E, 64);
+  if (E_pad > 128) return cudaErrorInvalidValue;
+  int n_xst = 4;
+  while (n_xst > 2 && bwd_layout(E_pad, n_xst, p.dm.K).total > 227u * 1024u) --n_xst;
+  const uint32_t smem = bwd_layout(E_pad, n_xst, p.dm.K).total;
+  if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
+  cudaError_t e = cudaFuncSetAttribute(k_router_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_router_bwd_tc<<<p.groups * p.slices, 320, smem, s>>>(tmX, tmW, tmDX, p, E_pad, n_xst);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s) {
+  if (p.dm.E > kF32MaxE) return cudaErrorInvalidValue;
+  const size_t smem = sizeof(float) * 64 * (p.dm.E + 1);
+  k_router_bwd_f32<<<p.n_tiles, 256, smem, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s) {
+  const size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
+  const int threads = 256;
+  const int blocks = static_cast<int>((n + threads - 1) / threads);
+  k_dw_reduce<<<blocks, threads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace smoes

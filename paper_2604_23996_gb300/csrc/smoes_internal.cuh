@@ -1,0 +1,169 @@
+// smoes_internal.cuh -- types shared by the host API (api.cu) and the kernels.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "smoes.h"
+
+namespace smoes {
+
+constexpr int kMaxTopK = 16;
+constexpr int kMaxBins = 32;
+constexpr int kMaxExperts = 256;
+constexpr int kPieceTokens = 32;           // one warp of tokens per partial-sum "piece"
+constexpr uint32_t kStatusData = 1u;       // status word bits
+constexpr uint32_t kStatusTimeout = 2u;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s for any bounded device wait
+
+// Values accumulated per piece (a warp's tokens of one sample), in this order:
+//   Q[k] = sum p_jk, Rv[k] = sum dv_j p_jk, Rt[k] = sum dt_j p_jk, Nv[k] = sum Mv_j p_jk,
+//   Nt[k] = sum Mt_j p_jk, then Dv = sum dv_j, Dt = sum dt_j, Av = sum Mv_j, At = sum Mt_j,
+// where dm_j = M_jm - 1/2. The centred sums carry the modality/bin covariance without
+// cancellation when M is close to 1/2 (the Gaussian score at tau = 0.5 d); the direct sums
+// stay accurate when a modality's mass is small.
+__host__ __device__ constexpr int piece_values(int K) { return 5 * K + 4; }
+__host__ __device__ constexpr int piece_stride(int K) { return (piece_values(K) + 3) & ~3; }
+
+// Device view of the caller-owned workspace (all pointers inside one allocation).
+struct WsView {
+  uint32_t* status;          // [4]: status bits, absent-modality count, spare, spare
+  uint32_t* sample_ticket;   // [B] pieces completed per sample (self-resetting)
+  uint32_t* loss_ticket;     // [1] samples completed (self-resetting)
+  const int32_t* offsets;    // [B+1]
+  const int32_t* token_sample;   // [T]
+  const int32_t* expert_bin;     // [E]
+  const int32_t* expert_slot;    // [E]
+  const int32_t* piece_base;     // [n_groups+1] first piece of each 32-token group
+  const int32_t* sample_pieces;  // [B+1] pieces of sample i are [sp[i], sp[i+1])
+  float* pieces;             // [n_pieces * piece_stride]
+  double* mi64;              // [B]
+  float* tabs;               // [B * 3 * K]: a_k, b_k, h_k per sample (backward coefficients)
+  float* gsave;              // [T * E] softmax scores saved by the forward
+  float* dw_part;            // [G * E * d] per-token-group partial dW
+  int32_t* perm_scratch;     // permutation block counts / offsets
+  uint32_t* attn_ticket;     // [B * ceil(S/128)] head tickets of the attention score
+  float* attn_part;          // [H_max * T] per-head vision mass
+};
+
+struct Dims {
+  int T, d, E, k, K, B, N_B, renorm;
+  int pstride;               // piece_stride(K)
+  int n_groups;              // ceil(T / 32)
+};
+
+struct FwdParams {
+  Dims dm;
+  WsView ws;
+  const void* X;
+  const void* W;             // [E, d] (read directly by the fp32 path; bf16 goes through TMA)
+  const float* M_in;         // provided scores, or null when the Gaussian score is fused
+  const float* mu;           // [2, d] (Gaussian mode)
+  const float* var;          // [2, d]
+  float inv_tau;
+  float* M_out;
+  int32_t* topk_idx;
+  float* topk_w;
+  float* bin_prob;
+  float* joint;
+  float* mi;
+  float* loss;
+  int n_tiles;
+  uint64_t limit_ns;
+};
+
+struct BwdParams {
+  Dims dm;
+  WsView ws;
+  const void* X;
+  const void* W;
+  const float* M;
+  const int32_t* topk_idx;
+  const float* d_topk_w;
+  float scale;               // -loss_scale / B
+  void* dX;
+  float* dlogits;
+  float* dW;
+  int accumulate;
+  int groups;                // G token groups (partial dW blocks)
+  int slices;                // d-slices per token group (tcgen05 path)
+  int slice_width;           // columns per d-slice
+  int n_tiles;               // token tiles
+  uint64_t limit_ns;
+};
+
+struct PermParams {
+  int T, k, E, K;
+  const int32_t* topk_idx;
+  const int32_t* home;
+  const uint8_t* is_vision;
+  const int32_t* expert_bin;
+  const int32_t* expert_slot;
+  int32_t* bin_offsets;
+  int32_t* perm_token;
+  uint32_t* perm_mask;
+  int32_t* dispatch;
+  int32_t* expert_counts;
+  int32_t* blk_counts;       // [n_blocks * K]
+  int32_t* blk_offsets;      // [n_blocks * K]
+  uint32_t* status;
+  int n_blocks;
+};
+
+struct GaussParams {
+  int T, d;
+  const void* X;
+  const float* mu;
+  const float* var;
+  float inv_tau;
+  float* M;
+  uint32_t* status;
+};
+
+struct AttnParams {
+  int B, H, S, hd, T;
+  const void* Q;
+  const void* K;
+  const uint8_t* is_vision;
+  const float* m_prev;
+  const float* key_bias;
+  float scale_log2;          // sm_scale * log2(e)
+  int causal;
+  const float* xattn_norm;
+  const float* x_norm;
+  float* M;
+  float* part;               // [H * T]
+  uint32_t* ticket;          // [B * n_qtiles]
+  uint32_t* status;
+  int n_qtiles;
+  int n_items;
+  uint64_t limit_ns;
+};
+
+// ------------------------------------------------------------------ launchers (in .cu files)
+cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
+                                   const CUtensorMap& tmW, int n_sms, cudaStream_t s);
+cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s);
+cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX,
+                                   const CUtensorMap& tmW, const CUtensorMap& tmDX,
+                                   cudaStream_t s);
+cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s);
+cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s);
+cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s);
+cudaError_t launch_gauss_score(const GaussParams& p, smoes_dtype dt, int n_sms, cudaStream_t s);
+cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+                             int n_sms, cudaStream_t s);
+
+// Shape helpers shared by host and device code.
+__host__ __device__ constexpr int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+// Forward (tcgen05): 128-token tiles, K-blocks of 64 bf16 (128-byte rows).
+constexpr int kFwdBM = 128;
+constexpr int kFwdBK = 64;
+// Backward (tcgen05): 64-token tiles, 128-column d-blocks.
+constexpr int kBwdBT = 64;
+constexpr int kBwdBD = 128;
+
+}  // namespace smoes

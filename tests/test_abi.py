@@ -1,0 +1,79 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds and loads, exports every
+entry point include/smoes.h declares, and plan creation validates its arguments."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def bd():
+    from paper_2604_23996_gb300.build import build_library
+    build_library()
+    from paper_2604_23996_gb300 import binding
+    return binding
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "smoes.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(smoes_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_four_path_calls():
+    fns = declared_functions()
+    for name in ("smoes_router_fwd", "smoes_router_bwd", "smoes_modality_score", "smoes_bin_permute"):
+        assert name in fns
+
+
+def test_library_exports_every_declared_symbol(bd):
+    import ctypes
+    lib = ctypes.CDLL(bd.LIB)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(declared_functions()) == set(bd.exported_symbols())
+
+
+def _plan(bd, **kw):
+    args = dict(T=100, d=64, E=16, k=2, n_bins=4, sample_offsets=[0, 40, 100],
+                expert_bin=np.arange(16) // 4, dtype=bd.SMOES_BF16)
+    args.update(kw)
+    return bd.smoes_plan_create(**args)
+
+
+def test_plan_create_ok_and_workspace_size(bd):
+    code, plan = _plan(bd)
+    assert code == 0
+    n = bd.smoes_workspace_bytes(plan)
+    assert n > 100 * 16 * 4            # at least the saved softmax scores
+    bd.smoes_plan_destroy(plan)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(d=60), -1),                                        # d % 8 != 0
+    (dict(k=17, E=32, expert_bin=np.arange(32) // 8), -2),   # k > 16
+    (dict(E=18, expert_bin=np.arange(18) % 4), -1),          # E % n_bins != 0
+    (dict(sample_offsets=[0, 40, 90]), -1),                  # o_B != T
+    (dict(sample_offsets=[0, 40, 40, 100]), -1),             # empty sample
+    (dict(expert_bin=np.array([0] * 5 + [1] * 3 + [2] * 4 + [3] * 4)), -1),   # unequal bins
+    (dict(expert_bin=np.arange(16) // 4 + 1), -1),           # bin out of range
+    (dict(n_bins=64, E=64, expert_bin=np.arange(64)), -2),   # more than 32 bins
+    (dict(k=0), -1),
+])
+def test_plan_create_rejects(bd, kw, code):
+    got, plan = _plan(bd, **kw)
+    assert got == code
+
+
+def test_empty_batch_plan(bd):
+    code, plan = bd.smoes_plan_create(0, 64, 16, 2, 4, [0], np.arange(16) // 4, bd.SMOES_BF16)
+    assert code == 0
+    bd.smoes_plan_destroy(plan)
+
+
+def test_status_strings(bd):
+    assert bd.smoes_status_string(0) == "ok"
+    assert "workspace" in bd.smoes_status_string(-4)
