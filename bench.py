@@ -1,0 +1,411 @@
+#!/usr/bin/env python
+"""Router fwd+bwd throughput of the SMoES hot path on GB300 (one JSON line on stdout).
+
+A step is one pass of the whole router hot path over one batch of the workload:
+  smoes_router_fwd (gate GEMM + Gaussian modality score + softmax/top-k/bins + per-sample MI)
+  -> smoes_router_bwd (MI gradient -> dW and dX) -> smoes_bin_permute (de-duplicated dispatch).
+Default workload: the DeepSeekMoE-style VLM layer, T = 16384 tokens (8 x [576 image + 1472 text]),
+d = 2048, E = 64 routed experts, top-6, 8 bins, bf16. Inputs are seeded synthetic data.
+
+Timing: W warm-up steps, then K timed steps. Each call is replayed from a CUDA graph; before
+every step the L2 is flushed by writing a 256 MiB buffer (outside the timed interval), and CUDA
+events on the launching stream bracket each call. --gpus N under torchrun runs N independent
+replicas (the path needs no collective); time = max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "router fwd+bwd tokens/sec per MoE layer on 1 GB300; % of HBM/tensor roofline"
+UNIT = "tokens/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="dsmoe_vlm")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--profile", action="store_true",
+                    help="short run for ncu: no clock load window, no e2e, no CPU baseline")
+    args = ap.parse_args()
+    if args.profile:
+        args.no_e2e = args.no_cpu_baseline = True
+    return args
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), float(p["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+WORKLOAD_TEXT = {
+    "tiny_fp32": "T=4096 (2458 img + 1638 txt, 1 sample), d=512, E=16 top-2, 4 bins, fp32",
+    "dsmoe_vlm": "T=16384 (8x[576 img + 1472 txt]), d=2048, E=64 top-6, 8 bins, bf16",
+    "small_hidden": "T=32768 (16x[729 img + 1319 txt]), d=1280, E=64 top-6, 8 bins, bf16",
+    "attn_router": "T=32768 (8x[1024 img + 3072 txt]), d=2048, E=64 top-6, 8 bins, bf16",
+    "large_fine": "T=131072 (32x[1024 img + 3072 txt]), d=2048, E=128 top-8, 16 bins, bf16",
+}
+
+
+def algorithmic(wl):
+    """Algorithmic bytes and flops of one step and of the backward call (the dominant launch)."""
+    T, d, E, k, K = wl.T, wl.d, wl.E, wl.k, wl.n_bins
+    b = wl.X.element_size()
+    per_token = 3 * d * b + 8 * k + 16 + 4 * k + 8 * min(k, K)
+    step_bytes = T * per_token + E * d * (b + 4)
+    step_flops = 6.0 * T * d * E
+    bwd_bytes = T * (2 * d * b + 8) + E * d * (b + 4)        # X read, dX write, M read, W read, dW write
+    return step_bytes, step_flops, bwd_bytes, 4.0 * T * d * E
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        if vis:
+            try:
+                gpu_index = int(vis.split(",")[gpu_index])
+            except (ValueError, IndexError):
+                pass
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def wait_first(self, timeout=5.0):
+        t0 = time.time()
+        while self.proc is not None and not self.lines and time.time() - t0 < timeout:
+            time.sleep(0.02)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        out = {"sm_mhz": float(np.median(sm)) if sm else None,
+               "sm_max_mhz": float(max(smax)) if smax else None,
+               "reasons": sorted(reasons), "samples": len(sm)}
+        if not sm and self.proc is not None:
+            out["error"] = (self.proc.stderr.read() or "")[:200]
+        return out
+
+
+def profile_traffic(kernel_file, workload):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on the current source."""
+    path = os.path.join(ROOT, "profiles", f"traffic_{workload}.json")
+    src = os.path.join(ROOT, "paper_2604_23996_gb300", "csrc", kernel_file)
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        if rec.get("source_sha") == sha:
+            return float(rec["dram_bytes_per_launch"])
+    except Exception:
+        pass
+    return None
+
+
+def cpu_oracle_rate(wl, budget_s=10.0):
+    """Oracle (fp64 numpy) fwd + bwd + permutation on whole samples of the workload, until the
+    time budget is used (at least one sample). Returns (tokens/s, samples, tokens, seconds)."""
+    from oracle import smoes_oracle as O
+    offs = wl.sample_offsets
+    Xd_all = wl.X
+    mu = wl.mu.double().numpy()
+    var = wl.var.double().numpy()
+    Wd = wl.W.double().numpy()
+    done_tok, t_used, n = 0, 0.0, 0
+    for it in range(10 ** 6):
+        i = it % wl.B
+        s, e = int(offs[i]), int(offs[i + 1])
+        Xd = Xd_all[s:e].double().numpy()
+        t0 = time.perf_counter()
+        M = O.gaussian_score(Xd, mu, var, wl.tau)
+        one = np.array([0, e - s])
+        fwd = O.router_forward(Xd, Wd, M, wl.expert_bin, wl.n_bins, one, wl.k)
+        O.router_backward(Xd, Wd, M, fwd, wl.expert_bin, one, 1.0)
+        O.bin_permute(fwd["topk_idx"], wl.expert_bin, wl.n_bins, is_vision=wl.is_vision[s:e])
+        t_used += time.perf_counter() - t0
+        done_tok += e - s
+        n += 1
+        if t_used >= budget_s:
+            break
+    return done_tok / t_used, n, done_tok, t_used
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def run_reference(args, rank, world):
+    """The reference arm: the fp64 oracle on the host cores, one bounded sample per step."""
+    from paper_2604_23996_gb300.workloads import config_workload
+    if rank != 0:
+        return
+    wl = config_workload(args.config)
+    for _ in range(args.warmup):
+        cpu_oracle_rate(wl, budget_s=0.0)
+    t_tot, tok = 0.0, 0
+    for _ in range(args.steps):
+        rate, n, ntok, secs = cpu_oracle_rate(wl, budget_s=0.0)
+        t_tot += secs
+        tok += ntok
+    value = tok / t_tot
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * t_tot / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "impl": "reference",
+            "config": {"workload": f"{args.config}: {WORKLOAD_TEXT[args.config]}",
+                       "sample": "one sample (first of the batch) per step"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle",
+                             "sample": f"{tok // args.steps} tokens (one sample) per step"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    from paper_2604_23996_gb300 import binding as bd
+    from paper_2604_23996_gb300.workloads import config_workload
+
+    wl = config_workload(args.config)
+    dtype = bd.SMOES_BF16 if wl.dtype == torch.bfloat16 else bd.SMOES_F32
+    r = bd.Router(wl.T, wl.d, wl.E, wl.k, wl.n_bins, wl.sample_offsets, wl.expert_bin, dtype)
+    X = wl.X.to(dev)
+    W = wl.W.to(dev)
+    mu, var = wl.mu.to(dev), wl.var.to(dev)
+    is_vis = torch.from_numpy(wl.is_vision).to(dev)
+    dW = torch.empty((wl.E, wl.d), dtype=torch.float32, device=dev)
+    dX = torch.empty_like(X)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)   # 256 MiB > L2
+
+    def fwd():
+        r.forward(X, W, mu=mu, var=var, tau=wl.tau, bin_prob=False)
+
+    def bwd():
+        r.backward(X, W, r.M, dW, dX=dX, loss_scale=1e-4)
+
+    def perm():
+        r.permute(is_vision=is_vis)
+
+    # eager warm-up (also checks the device status once), then graph capture per call
+    for _ in range(2):
+        fwd(); bwd(); perm()
+    code, _ = r.device_status()
+    assert code == 0, f"device status {code}"
+    graphs = []
+    s = torch.cuda.Stream(device=dev)
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        for fn in (fwd, bwd, perm):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                fn()
+            graphs.append(g)
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    launches_per_step = 6          # fwd 1, bwd 2 (main + dW reduce), permutation 3
+
+    def step_timed():
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ev[0].record()
+        graphs[0].replay()
+        ev[1].record()
+        graphs[1].replay()
+        ev[2].record()
+        graphs[2].replay()
+        ev[3].record()
+        return ev
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step_timed()
+    torch.cuda.synchronize()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    # clocks: sampled from a load window that starts ~0.5 s before the timed steps (the timed
+    # steps alone last a few ms, shorter than the sampling period) and ends after them
+    clocks = ClockSampler(local)
+    if not args.profile:
+        clocks.start()
+        clocks.wait_first()
+        t_load = time.time()
+        while time.time() - t_load < 0.5:
+            flush.zero_()
+            step_timed()
+            torch.cuda.synchronize()
+    evs = []
+    for _ in range(args.steps):
+        flush.zero_()
+        evs.append(step_timed())
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clk = clocks.stop() if not args.profile else {"sm_mhz": None, "note": "profile run"}
+    t_step = [e[0].elapsed_time(e[3]) for e in evs]
+    t_fwd = [e[0].elapsed_time(e[1]) for e in evs]
+    t_bwd = [e[1].elapsed_time(e[2]) for e in evs]
+    t_perm = [e[2].elapsed_time(e[3]) for e in evs]
+    total_ms = float(np.sum(t_step))
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = world * wl.T / (ms_per_step * 1e-3)
+
+    # end to end through the public API: host inputs in pinned memory, copies inside the region
+    e2e = None
+    if not args.no_e2e:
+        Xh = wl.X.pin_memory()
+        Wh = wl.W.pin_memory()
+        muh, varh = wl.mu.pin_memory(), wl.var.pin_memory()
+        lossh = torch.empty(1, dtype=torch.float32).pin_memory()
+        h2d = (Xh.numel() * Xh.element_size() + Wh.numel() * Wh.element_size() +
+               muh.numel() * 4 + varh.numel() * 4)
+        d2h = 4
+
+        def e2e_step():
+            X.copy_(Xh, non_blocking=True)
+            W.copy_(Wh, non_blocking=True)
+            mu.copy_(muh, non_blocking=True)
+            var.copy_(varh, non_blocking=True)
+            fwd(); bwd(); perm()
+            lossh.copy_(r.loss, non_blocking=True)
+
+        for _ in range(3):
+            flush.zero_()
+            e2e_step()
+        torch.cuda.synchronize()
+        t_e2e = 0.0
+        for _ in range(args.steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            e2e_step()
+            b.record()
+            b.synchronize()
+            t_e2e += a.elapsed_time(b)
+        e2e = {"value": world * wl.T / (t_e2e / args.steps * 1e-3), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    hbm, tf_burst, tf_sus, peak_kind = peaks()
+    step_bytes, step_flops, bwd_bytes, bwd_flops = algorithmic(wl)
+    bwd_ms = float(np.mean(t_bwd))
+    achieved = bwd_bytes / (bwd_ms * 1e-3) / 1e9
+    t_roof = max(step_bytes / (hbm * 1e9), step_flops / (tf_sus * 1e12))
+    traffic = profile_traffic("router_bwd.cu", args.config)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == torch.bfloat16 else "f32",
+        "data": "synthetic (seeded; shapes of the paper's MoE-VLM router layers)",
+        "config": {"workload": f"{args.config}: {WORKLOAD_TEXT[args.config]}; Gaussian score; "
+                               "fwd + bwd (dW, dX) + bin permutation",
+                   "l2": "flushed before every step (256 MiB write, outside the timed interval)",
+                   "clocks": "nvidia-smi every 100 ms over a load window of ~0.5 s of steps "
+                             "ending with the timed steps",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
+                     "kernel": "smoes_router_bwd (k_router_bwd_tc + k_dw_reduce)",
+                     "peak_source": peak_kind},
+        "step_roofline": {"t_roof_us": t_roof * 1e6, "t_step_us": ms_per_step * 1e3,
+                          "frac": t_roof / (ms_per_step * 1e-3),
+                          "bytes": step_bytes, "flops": step_flops},
+        "breakdown_us": {"fwd": 1e3 * float(np.mean(t_fwd)), "bwd": 1e3 * bwd_ms,
+                         "permute": 1e3 * float(np.mean(t_perm))},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if not args.no_cpu_baseline and world == 1:
+        rate, n, ntok, secs = cpu_oracle_rate(wl)
+        line["cpu_baseline"] = {"value": rate, "unit": UNIT, "cores": cores(), "kind": "oracle",
+                                "sample": f"{n} whole samples of {wl.B} ({ntok} tokens, repeated), {secs:.1f} s"}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

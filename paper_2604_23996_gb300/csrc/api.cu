@@ -11,6 +11,7 @@
 
 namespace smoes {
 int perm_blocks(int T);
+int perm_rounds(int T);
 }
 
 using namespace smoes;
@@ -22,7 +23,7 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
   size_t status, sample_ticket, loss_ticket, offsets, token_sample, expert_bin, expert_slot,
-      piece_base, sample_pieces, pieces, mi64, tabs, gsave, dw_part, perm, attn_ticket, attn_part;
+      piece_base, sample_pieces, pieces, mi32, tabs, gsave, dw_part, dz_img, perm, attn_ticket, attn_part;
   size_t header_bytes;   // [0, header_bytes) is cleared by smoes_workspace_init
   size_t total;
 };
@@ -32,7 +33,7 @@ struct Layout {
 struct smoes_plan_s {
   smoes_router_desc desc{};
   int N_B = 1;
-  int n_groups = 0;      // ceil(T / 32)
+  int n_groups = 0;      // ceil(T / 128): forward tiles, one partial-sum piece per (tile, sample)
   int n_pieces = 0;
   int n_sms = 148;
   // backward decomposition
@@ -61,10 +62,11 @@ WsView make_view(const smoes_plan_s* P, void* ws) {
   v.piece_base = reinterpret_cast<const int32_t*>(b + L.piece_base);
   v.sample_pieces = reinterpret_cast<const int32_t*>(b + L.sample_pieces);
   v.pieces = reinterpret_cast<float*>(b + L.pieces);
-  v.mi64 = reinterpret_cast<double*>(b + L.mi64);
+  v.mi32 = reinterpret_cast<float*>(b + L.mi32);
   v.tabs = reinterpret_cast<float*>(b + L.tabs);
   v.gsave = reinterpret_cast<float*>(b + L.gsave);
   v.dw_part = reinterpret_cast<float*>(b + L.dw_part);
+  v.dz_img = b + L.dz_img;
   v.perm_scratch = reinterpret_cast<int32_t*>(b + L.perm);
   v.attn_ticket = reinterpret_cast<uint32_t*>(b + L.attn_ticket);
   v.attn_part = reinterpret_cast<float*>(b + L.attn_part);
@@ -252,10 +254,12 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.piece_base = take(sizeof(int32_t) * (P->n_groups + 1));
   L.sample_pieces = take(sizeof(int32_t) * (B + 1));
   L.pieces = take(sizeof(float) * static_cast<size_t>(std::max(P->n_pieces, 1)) * piece_stride(K));
-  L.mi64 = take(sizeof(double) * std::max(B, 1));
+  L.mi32 = take(sizeof(float) * std::max(B, 1));
   L.tabs = take(sizeof(float) * 3 * K * static_cast<size_t>(std::max(B, 1)));
   L.gsave = take(sizeof(float) * static_cast<size_t>(T) * E);
   L.dw_part = take(sizeof(float) * static_cast<size_t>(P->bwd_groups) * E * d.d);
+  L.dz_img = take(d.dtype == SMOES_BF16 && E <= 128
+                      ? static_cast<size_t>(P->bwd_tiles) * 2 * round_up(E, 64) * 128 : 0);
   L.perm = take(sizeof(int32_t) * 2 * static_cast<size_t>(P->perm_nblocks) * K);
   L.attn_part = take(sizeof(float) * static_cast<size_t>(T) * std::max(0, d.attn_max_heads));
   L.total = o;
@@ -466,7 +470,8 @@ smoes_status smoes_router_bwd(smoes_plan P, const void* X, const void* W, const 
     } else {
       tdx = tx;   // unused
     }
-    e = launch_router_bwd_bf16(p, tx, tw, tdx, stream);
+    e = launch_dz_prep(p, stream);
+    if (e == cudaSuccess) e = launch_router_bwd_bf16(p, tx, tw, tdx, stream);
   } else {
     e = launch_router_bwd_f32(p, stream);
   }
@@ -511,6 +516,7 @@ smoes_status smoes_bin_permute(smoes_plan P, const int32_t* topk_idx, const int3
   p.blk_offsets = v.perm_scratch + static_cast<size_t>(P->perm_nblocks) * d.n_bins;
   p.status = v.status;
   p.n_blocks = P->perm_nblocks;
+  p.rounds = perm_rounds(d.T);
   return cuda_status(launch_bin_permute(p, stream));
 }
 

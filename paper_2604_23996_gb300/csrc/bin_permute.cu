@@ -13,9 +13,7 @@
 namespace smoes {
 namespace {
 
-constexpr int kPermThreads = 256;
-constexpr int kPermRounds = 4;                        // tokens per block = 1024
-constexpr int kPermTokens = kPermThreads * kPermRounds;
+constexpr int kPermThreads = 256;                    // one token per thread and round
 
 struct TokenSel {
   int e[kMaxTopK];
@@ -46,8 +44,8 @@ __global__ void __launch_bounds__(kPermThreads) k_perm_count(const PermParams p)
   __shared__ int wc[kPermThreads / 32][kMaxBins];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int cnt = 0;                                          // lane kb of each warp counts bin kb
-  for (int r = 0; r < kPermRounds; ++r) {
-    const int j = blockIdx.x * kPermTokens + r * kPermThreads + threadIdx.x;
+  for (int r = 0; r < p.rounds; ++r) {
+    const int j = (blockIdx.x * p.rounds + r) * kPermThreads + threadIdx.x;
     TokenSel s;
     s.bins = 0u;
     if (j < p.T) load_sel(p, j, s);
@@ -126,8 +124,8 @@ __global__ void __launch_bounds__(kPermThreads) k_perm_scatter(const PermParams 
   if (threadIdx.x < p.K) base[threadIdx.x] = p.blk_offsets[blockIdx.x * p.K + threadIdx.x];
   __syncthreads();
   const unsigned lt_mask = (1u << lane) - 1u;
-  for (int r = 0; r < kPermRounds; ++r) {
-    const int j = blockIdx.x * kPermTokens + r * kPermThreads + threadIdx.x;
+  for (int r = 0; r < p.rounds; ++r) {
+    const int j = (blockIdx.x * p.rounds + r) * kPermThreads + threadIdx.x;
     const bool valid = j < p.T;
     TokenSel s;
     s.bins = 0u;
@@ -186,7 +184,16 @@ __global__ void __launch_bounds__(kPermThreads) k_perm_scatter(const PermParams 
 
 }  // namespace
 
-int perm_blocks(int T) { return (T + kPermTokens - 1) / kPermTokens; }
+// Rounds of 256 tokens per block: 1 while that keeps the block count <= 1024 (the scan runs in
+// one block of 1024 threads), more for larger batches.
+int perm_rounds(int T) {
+  const int units = (T + kPermThreads - 1) / kPermThreads;
+  return units <= 1024 ? 1 : (units + 1023) / 1024;
+}
+int perm_blocks(int T) {
+  const int per = kPermThreads * perm_rounds(T);
+  return (T + per - 1) / per;
+}
 
 cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s) {
   if (p.n_blocks > 1024) return cudaErrorInvalidValue;

@@ -7,15 +7,17 @@
 // gradient of the top-k weights is pushed through the (renormalised) softmax as well.
 // Then dW = dz^T X and dX = dz W.
 //
-// tcgen05 path (bf16): CTA (token group g, d-slice s). Per 64-token tile, four "dz" warps build
-// dz in shared memory as a bf16 hi/lo pair (dz = hi + lo to ~2^-17 relative), and one thread
-// issues, per 128-column d-block of the slice,
+// tcgen05 path (bf16): k_dz_prep writes dz of every 64-token tile as a bf16 hi/lo pair
+// (dz = hi + lo to ~2^-17 relative) directly in the 128-byte-swizzled shared-memory image the
+// tensor cores read. The main kernel runs CTA (token group g, d-slice s): per tile it bulk-copies
+// that image, and one thread issues, per 128-column d-block of the slice,
 //   dW^T[d-block] += X^T(tile) . dz        (M = 128 d, N = E_pad, K = 64 tokens)  -> TMEM, kept
 //   dX^T[d-block]  = W^T(d-block) . dz^T   (M = 128 d, N = 64 tokens, K = E_pad)  -> TMEM, drained
 // X tiles arrive by TMA; the W slice stays resident in shared memory; dX leaves by TMA store.
 // The per-group dW^T slice is written once at the end and summed over groups in fixed order.
 #include <cuda_bf16.h>
 
+#include "device_common.cuh"
 #include "ptx.cuh"
 #include "smoes_internal.cuh"
 
@@ -80,40 +82,118 @@ __device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
   return r;
 }
 
+// ------------------------------------------------------------------ dz preparation (bf16 path)
+// TPT = E_pad/8 threads per token, 8 experts each; the token's sum over experts is a shuffle
+// reduction inside its TPT-lane group. Rows beyond T and padded experts are written as zeros.
+template <int TPT>
+__global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
+  const Dims& dm = p.dm;
+  const int E = dm.E, K = dm.K, k = dm.k;
+  constexpr int kEp = TPT * 8;
+  const int j = (blockIdx.x * 256 + threadIdx.x) / TPT;
+  const int c = threadIdx.x % TPT;
+  const int e0 = c * 8;
+  const int n_rows = p.n_tiles * kBwdBT;
+  if (j >= n_rows) return;                            // whole TPT groups exit together
+  const bool valid = j < dm.T;
+  float g[8], u[8];
+  float dv = 0.f, dt = 0.f;
+  if (valid) {
+    const float* grow = p.ws.gsave + static_cast<size_t>(j) * E;
+    if ((E & 3) == 0 && e0 + 8 <= E) {
+      const float4 a = __ldcg(reinterpret_cast<const float4*>(grow + e0));
+      const float4 b = __ldcg(reinterpret_cast<const float4*>(grow + e0 + 4));
+      g[0] = a.x; g[1] = a.y; g[2] = a.z; g[3] = a.w; g[4] = b.x; g[5] = b.y; g[6] = b.z; g[7] = b.w;
+    } else {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) g[q] = (e0 + q < E) ? __ldcg(grow + e0 + q) : 0.f;
+    }
+    const float2 m = __ldg(reinterpret_cast<const float2*>(p.M) + j);
+    dv = m.x - 0.5f;
+    dt = m.y - 0.5f;
+    const float* tb = p.ws.tabs + static_cast<size_t>(p.ws.token_sample[j]) * 3 * K;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      u[q] = 0.f;
+      if (e0 + q < E) {
+        const int b = __ldg(p.ws.expert_bin + e0 + q);
+        u[q] = __ldcg(tb + 2 * K + b) + dv * __ldcg(tb + b) + dt * __ldcg(tb + K + b);
+      }
+    }
+  } else {
+#pragma unroll
+    for (int q = 0; q < 8; ++q) { g[q] = 0.f; u[q] = 0.f; }
+  }
+  float part = 0.f;
+#pragma unroll
+  for (int q = 0; q < 8; ++q) part = fmaf(g[q], u[q], part);
+#pragma unroll
+  for (int o = 1; o < TPT; o <<= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+  float dz[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) dz[q] = p.scale * g[q] * (u[q] - part);
+  if (valid && p.d_topk_w != nullptr) {
+    Upstream up;
+    load_upstream(p, j, up);
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      if (e0 + q < E) dz[q] += g[q] * (upstream_at(up, k, e0 + q) - up.gdt);
+  }
+  if (valid && p.dlogits) {
+    float* dl = p.dlogits + static_cast<size_t>(j) * E;
+    if ((E & 3) == 0 && e0 + 8 <= E) {
+      *reinterpret_cast<float4*>(dl + e0) = make_float4(dz[0], dz[1], dz[2], dz[3]);
+      *reinterpret_cast<float4*>(dl + e0 + 4) = make_float4(dz[4], dz[5], dz[6], dz[7]);
+    } else {
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (e0 + q < E) dl[e0 + q] = dz[q];
+    }
+  }
+  uint32_t hw[4], lw[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(dz[2 * q]), h1 = __float2bfloat16_rn(dz[2 * q + 1]);
+    hw[q] = static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
+    lw[q] = pack_bf16x2(dz[2 * q] - __bfloat162float(h0), dz[2 * q + 1] - __bfloat162float(h1));
+  }
+  const int tile = j / kBwdBT, r = j % kBwdBT;
+  uint8_t* img = p.ws.dz_img + static_cast<size_t>(tile) * (2 * kEp * 128);
+  const uint32_t off = (e0 >> 6) * 8192u + sw128_offset(static_cast<uint32_t>(r), static_cast<uint32_t>(e0 & 63));
+  *reinterpret_cast<uint4*>(img + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+  *reinterpret_cast<uint4*>(img + kEp * 128 + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+}
+
 // ------------------------------------------------------------------ tcgen05 backward (bf16)
 
 struct BwdLayout {
-  uint32_t wsl, dz, xst, stg, ubar, us, bars, total;
+  uint32_t wsl, dz, xst, stg, bars, total;
 };
 
-__host__ __device__ inline BwdLayout bwd_layout(int E_pad, int n_xst, int K) {
+__host__ __device__ inline BwdLayout bwd_layout(int E_pad, int n_xst) {
   BwdLayout L;
   uint32_t o = 0;
-  L.wsl = o;  o += 65536u;                                     // W slice (ds * E_pad * 2 B)
-  L.dz = o;   o += 2u * 2u * static_cast<uint32_t>(E_pad) * 128u; // 2 buffers x (hi, lo)
-  L.xst = o;  o += static_cast<uint32_t>(n_xst) * 16384u;     // X stages [2 atoms][64][128 B]
-  L.stg = o;  o += 2u * 16384u;                                // dX staging [64][128] bf16 x2
-  L.ubar = o; o += 2u * 2u * 64u * 4u;                         // [2 buf][2 half][64]
-  L.us = o;   o += static_cast<uint32_t>(K) * 128u * 4u;       // [K][128]
-  L.bars = o; o += 8u * (2u * n_xst + 18u) + 16u;
+  L.wsl = o;  o += 65536u;                                         // W slice (ds * E_pad * 2 B)
+  L.dz = o;   o += 2u * 2u * static_cast<uint32_t>(E_pad) * 128u;   // 2 buffers x (hi, lo)
+  L.xst = o;  o += static_cast<uint32_t>(n_xst) * 16384u;          // X stages [2 atoms][64][128 B]
+  L.stg = o;  o += 2u * 16384u;                                    // dX staging [64][128] bf16 x2
+  L.bars = o; o += 8u * (2u * n_xst + 16u) + 16u;
   L.total = o + 1024u;
   return L;
 }
 
-__global__ void __launch_bounds__(320, 1)
+template <int E_pad>
+__global__ void __launch_bounds__(192, 1)
 k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
-                const __grid_constant__ CUtensorMap tmDX, const BwdParams p, const int E_pad,
-                const int n_xst) {
+                const __grid_constant__ CUtensorMap tmDX, const BwdParams p, const int n_xst) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const Dims& dm = p.dm;
-  const BwdLayout L = bwd_layout(E_pad, n_xst, dm.K);
+  const BwdLayout L = bwd_layout(E_pad, n_xst);
   uint8_t* wsl = base + L.wsl;
   uint8_t* dzb = base + L.dz;               // buffer zb: hi at zb*2*E_pad*128, lo right after
   uint8_t* xst = base + L.xst;
   uint8_t* stg = base + L.stg;
-  float* ubar = reinterpret_cast<float*>(base + L.ubar);
-  float* us = reinterpret_cast<float*>(base + L.us);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
   uint64_t* xfull = bars;
   uint64_t* xempty = bars + n_xst;
@@ -124,10 +204,9 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   uint64_t* wfull = dz_full + 8;
   uint64_t* dw_full = dz_full + 9;
   uint64_t* drain = dz_full + 10;
-  uint64_t* ub_bar = dz_full + 11;            // [2] dz warps exchange half sums
-  uint64_t* stg_free = dz_full + 13;          // [2] staging buffer may be rewritten
-  uint64_t* stg_full = dz_full + 15;          // [2] staging buffer written
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dz_full + 18);
+  uint64_t* stg_free = dz_full + 11;          // [2] staging buffer may be rewritten
+  uint64_t* stg_full = dz_full + 13;          // [2] staging buffer written
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dz_full + 16);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -136,8 +215,8 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   const int d0 = sl * p.slice_width;
   const int nb = min(p.slice_width, round_up(dm.d - d0, kBwdBD)) / kBwdBD;   // d-blocks here
   const bool want_dx = p.dX != nullptr;
-  const uint32_t dz_buf_bytes = 2u * static_cast<uint32_t>(E_pad) * 128u;   // hi + lo
-  const uint32_t dz_half = static_cast<uint32_t>(E_pad) * 128u;             // one of hi / lo
+  constexpr uint32_t dz_half = static_cast<uint32_t>(E_pad) * 128u;         // one of hi / lo
+  constexpr uint32_t dz_buf_bytes = 2u * dz_half;                           // hi + lo
   WaitCtx wc{abort_flag, p.ws.status, p.limit_ns};
 
   if (threadIdx.x == 0) {
@@ -147,11 +226,10 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       mbar_init(xempty + i, 1);
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(dz_full + i, 128);
+      mbar_init(dz_full + i, 1);
       mbar_init(dz_empty + i, 1);
       mbar_init(dx_full + i, 1);
       mbar_init(dx_empty + i, 128);
-      mbar_init(ub_bar + i, 128);
       mbar_init(stg_free + i, 1);
       mbar_init(stg_full + i, 128);
     }
@@ -171,7 +249,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   const uint32_t tm_dx = tmem + 256u;          // two 64-column dX^T buffers after the dW^T blocks
 
   if (warp == 0) {
-    // -------------------------------------------------------------- TMA producer
+    // -------------------------------------------------------------- TMA / bulk-copy producer
     if (lane == 0) {
       bool ok = true;
       mbar_arrive_expect_tx(wfull, static_cast<uint32_t>(nb) * 2u * dz_half);
@@ -179,8 +257,16 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
         tma_load_2d(wsl + a * dz_half, &tmW, wfull, d0 + 64 * a, 0);
       int st = 0;
       uint32_t ph = 0;
-      long issued = 0;
-      for (int t = grp; t < p.n_tiles && ok; t += G) {
+      long issued = 0, dz_issued = 0;
+      int lt = 0;
+      for (int t = grp; t < p.n_tiles && ok; t += G, ++lt) {
+        const int zb = lt & 1;
+        const uint32_t zuse = static_cast<uint32_t>(lt >> 1);
+        if (!mbar_wait(dz_empty + zb, (zuse & 1u) ^ 1u, wc)) { ok = false; break; }
+        mbar_arrive_expect_tx(dz_full + zb, dz_buf_bytes);
+        bulk_load(dzb + zb * dz_buf_bytes, p.ws.dz_img + static_cast<size_t>(t) * dz_buf_bytes,
+                  dz_buf_bytes, dz_full + zb);
+        ++dz_issued;
         for (int b = 0; b < nb; ++b) {
           if (!mbar_wait(xempty + st, ph ^ 1u, wc)) { ok = false; break; }
           uint8_t* xs = xst + st * 16384;
@@ -195,9 +281,11 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       int dummy = 0;
       wd.abort_flag = &dummy;
       mbar_wait(wfull, 0, wd);                // the W slice copy must land before exit
-      if (!ok) {
+      if (!ok) {                              // so must every issued X and dz copy
         for (long q = (issued > n_xst ? issued - n_xst : 0); q < issued; ++q)
           mbar_wait(xfull + (q % n_xst), static_cast<uint32_t>((q / n_xst) & 1), wd);
+        for (long q = (dz_issued > 2 ? dz_issued - 2 : 0); q < dz_issued; ++q)
+          mbar_wait(dz_full + (q & 1), static_cast<uint32_t>((q >> 1) & 1), wd);
       }
     }
   } else if (warp == 1) {
@@ -235,6 +323,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
             tc_fence_after();
             const uint32_t dxc = tm_dx + static_cast<uint32_t>(xb * kBwdBT);
             const uint32_t wa = smem_u32(wsl + 2 * b * dz_half);
+#pragma unroll
             for (int ke = 0; ke < E_pad / 16; ++ke) {    // K = 16 experts per instruction
               const uint64_t da = sdesc_sw128(wa + ke * 2048, dz_half, 1024);
               const uint32_t boff = (ke >> 2) * 8192 + (ke & 3) * 32;
@@ -259,7 +348,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       wd.abort_flag = &dummy;
       mbar_wait(drain, 0, wd);
     }
-  } else if (warp < 6) {
+  } else {
     // -------------------------------------------------------------- dX epilogue + dW drain
     const int lg = warp & 3;
     const int etid = threadIdx.x - 64;                 // 0..127
@@ -284,11 +373,11 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
           const uint32_t ta = tm_dx + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(xb * kBwdBT);
           const int drow = lg * 32 + lane;
 #pragma unroll
-          for (int c = 0; c < kBwdBT / 16; ++c) {
-            float v[16];
-            tmem_ld16(ta + 16u * c, v);
+          for (int c = 0; c < kBwdBT / 32; ++c) {
+            float v[32];
+            tmem_ld32(ta + 32u * c, v);
 #pragma unroll
-            for (int q = 0; q < 16; ++q) sg[(c * 16 + q) * kBwdBD + drow] = __float2bfloat16_rn(v[q]);
+            for (int q = 0; q < 32; ++q) sg[(c * 32 + q) * kBwdBD + drow] = __float2bfloat16_rn(v[q]);
           }
           tc_fence_before();
           mbar_arrive(dx_empty + xb);
@@ -310,91 +399,18 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       for (int b = 0; b < nb; ++b) {
         const int drow = d0 + b * kBwdBD + lg * 32 + lane;
         const uint32_t ta = tmem + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(b * E_pad);
-        for (int c = 0; c < E_pad / 16; ++c) {
-          float v[16];
-          tmem_ld16(ta + 16u * c, v);
 #pragma unroll
-          for (int q = 0; q < 16; ++q) {
-            const int e = c * 16 + q;
+        for (int c = 0; c < E_pad / 32; ++c) {
+          float v[32];
+          tmem_ld32(ta + 32u * c, v);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) {
+            const int e = c * 32 + q;
             if (e < dm.E && drow < dm.d)
               p.ws.dw_part[(static_cast<size_t>(grp) * dm.E + e) * dm.d + drow] = v[q];
           }
         }
       }
-    }
-  } else {
-    // -------------------------------------------------------------- dz producers (4 warps)
-    const int w4 = warp - 6;
-    const int r = (w4 & 1) * 32 + lane;                // token row in the tile
-    const int h = w4 >> 1;                             // expert half
-    const int dtid = threadIdx.x - 192;                // 0..127
-    const int Eh = E_pad / 2;
-    const int K = dm.K, E = dm.E, k = dm.k;
-    const float* gs = p.ws.gsave;
-    int lt = 0;
-    for (int t = grp; t < p.n_tiles; t += G, ++lt) {
-      const int zb = lt & 1;
-      const uint32_t zuse = static_cast<uint32_t>(lt >> 1);
-      if (!mbar_wait(dz_empty + zb, (zuse & 1u) ^ 1u, wc)) break;
-      const int j = t * kBwdBT + r;
-      const bool valid = j < dm.T;
-      float dv = 0.f, dt = 0.f;
-      if (valid) {
-        const int s = p.ws.token_sample[j];
-        const float2 m = *reinterpret_cast<const float2*>(p.M + 2 * static_cast<size_t>(j));
-        dv = m.x - 0.5f;
-        dt = m.y - 0.5f;
-        const float* tb = p.ws.tabs + static_cast<size_t>(s) * 3 * K;
-        for (int kb = 0; kb < K; ++kb)
-          us[kb * 128 + dtid] = __ldcg(tb + 2 * K + kb) + dv * __ldcg(tb + kb) + dt * __ldcg(tb + K + kb);
-      }
-      Upstream up;
-      const bool has_up = valid && p.d_topk_w != nullptr;
-      if (has_up) load_upstream(p, j, up);
-      // partial  sum_e g_e u_b(e)  over this thread's experts
-      float part = 0.f;
-      const int e0 = h * Eh;
-      for (int e = e0; e < e0 + Eh; ++e) {
-        if (valid && e < E) part += __ldcg(gs + static_cast<size_t>(j) * E + e) * us[p.ws.expert_bin[e] * 128 + dtid];
-      }
-      ubar[(zb * 2 + h) * 64 + r] = part;
-      mbar_arrive(ub_bar + zb);
-      if (!mbar_wait(ub_bar + zb, zuse & 1u, wc)) break;
-      const float ub = ubar[(zb * 2 + 0) * 64 + r] + ubar[(zb * 2 + 1) * 64 + r];
-      uint8_t* hib = dzb + zb * dz_buf_bytes;
-      uint8_t* lob = hib + dz_half;
-      for (int c = 0; c < Eh / 8; ++c) {
-        const int eb = e0 + c * 8;
-        float dz[8];
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const int e = eb + q;
-          float v = 0.f;
-          if (valid && e < E) {
-            const float g = __ldcg(gs + static_cast<size_t>(j) * E + e);
-            v = p.scale * g * (us[p.ws.expert_bin[e] * 128 + dtid] - ub);
-            if (has_up) v += g * (upstream_at(up, k, e) - up.gdt);
-          }
-          dz[q] = v;
-        }
-        if (valid && p.dlogits) {
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            if (eb + q < E) p.dlogits[static_cast<size_t>(j) * E + eb + q] = dz[q];
-        }
-        uint32_t hw[4], lw[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const __nv_bfloat16 h0 = __float2bfloat16_rn(dz[2 * q]), h1 = __float2bfloat16_rn(dz[2 * q + 1]);
-          hw[q] = static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
-          lw[q] = pack_bf16x2(dz[2 * q] - __bfloat162float(h0), dz[2 * q + 1] - __bfloat162float(h1));
-        }
-        const uint32_t off = (eb >> 6) * 8192u + sw128_offset(static_cast<uint32_t>(r), static_cast<uint32_t>(eb & 63));
-        *reinterpret_cast<uint4*>(hib + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-        *reinterpret_cast<uint4*>(lob + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-      }
-      fence_proxy_async_smem();
-      mbar_arrive(dz_full + zb);
     }
   }
 
@@ -489,14 +505,32 @@ k_router_bwd_f32(const BwdParams p) {
   }
 }
 
-// dW[e][c] = (accumulate ? dW[e][c] : 0) + sum_{g=0}^{G-1} part[g][e][c], in that order.
+// dW[e][c] = (accumulate ? dW[e][c] : 0) + S, S = sum_{g=0}^{G-1} part[g][e][c] in that order
+// (the group sum is formed first, so an existing dW adds one rounding, not G).
 __global__ void k_dw_reduce(const BwdParams p) {
   const size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
+  const size_t n4 = n / 4;
   const size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  float acc = p.accumulate ? p.dW[i] : 0.f;
-  for (int g = 0; g < p.groups; ++g) acc += __ldcg(p.ws.dw_part + static_cast<size_t>(g) * n + i);
-  p.dW[i] = acc;
+  if ((n & 3) == 0) {
+    if (i >= n4) return;
+    const float4* part = reinterpret_cast<const float4*>(p.ws.dw_part);
+    float4 acc = __ldcg(part + i);
+    for (int g = 1; g < p.groups; ++g) {
+      const float4 v = __ldcg(part + static_cast<size_t>(g) * n4 + i);
+      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    }
+    float4* dW = reinterpret_cast<float4*>(p.dW);
+    if (p.accumulate) {
+      const float4 o = dW[i];
+      acc.x += o.x; acc.y += o.y; acc.z += o.z; acc.w += o.w;
+    }
+    dW[i] = acc;
+  } else {
+    if (i >= n) return;
+    float acc = __ldcg(p.ws.dw_part + i);
+    for (int g = 1; g < p.groups; ++g) acc += __ldcg(p.ws.dw_part + static_cast<size_t>(g) * n + i);
+    p.dW[i] = p.accumulate ? p.dW[i] + acc : acc;
+  }
 }
 
 }  // namespace
@@ -505,13 +539,24 @@ cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, c
                                    const CUtensorMap& tmDX, cudaStream_t s) {
   const int E_pad = round_up(p.dm.E, 64);
   if (E_pad > 128) return cudaErrorInvalidValue;
-  int n_xst = 4;
-  while (n_xst > 2 && bwd_layout(E_pad, n_xst, p.dm.K).total > 227u * 1024u) --n_xst;
-  const uint32_t smem = bwd_layout(E_pad, n_xst, p.dm.K).total;
+  int n_xst = 6;
+  while (n_xst > 2 && bwd_layout(E_pad, n_xst).total > 227u * 1024u) --n_xst;
+  const uint32_t smem = bwd_layout(E_pad, n_xst).total;
   if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
-  cudaError_t e = cudaFuncSetAttribute(k_router_bwd_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto k = (E_pad == 64) ? k_router_bwd_tc<64> : k_router_bwd_tc<128>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_router_bwd_tc<<<p.groups * p.slices, 320, smem, s>>>(tmX, tmW, tmDX, p, E_pad, n_xst);
+  k<<<p.groups * p.slices, 192, smem, s>>>(tmX, tmW, tmDX, p, n_xst);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s) {
+  const int E_pad = round_up(p.dm.E, 64);
+  const long threads = static_cast<long>(p.n_tiles) * kBwdBT * (E_pad / 8);
+  const int blocks = static_cast<int>((threads + 255) / 256);
+  if (E_pad == 64) k_dz_prep<8><<<blocks, 256, 0, s>>>(p);
+  else if (E_pad == 128) k_dz_prep<16><<<blocks, 256, 0, s>>>(p);
+  else return cudaErrorInvalidValue;
   return cudaGetLastError();
 }
 
@@ -523,7 +568,8 @@ cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s) {
 }
 
 cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s) {
-  const size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
+  size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
+  if ((n & 3) == 0) n /= 4;
   const int threads = 256;
   const int blocks = static_cast<int>((n + threads - 1) / threads);
   k_dw_reduce<<<blocks, threads, 0, s>>>(p);

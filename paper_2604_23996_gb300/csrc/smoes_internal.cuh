@@ -13,7 +13,7 @@ namespace smoes {
 constexpr int kMaxTopK = 16;
 constexpr int kMaxBins = 32;
 constexpr int kMaxExperts = 256;
-constexpr int kPieceTokens = 32;           // one warp of tokens per partial-sum "piece"
+constexpr int kPieceTokens = 128;          // tokens per partial-sum "piece" (one forward tile)
 constexpr uint32_t kStatusData = 1u;       // status word bits
 constexpr uint32_t kStatusTimeout = 2u;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s for any bounded device wait
@@ -36,13 +36,14 @@ struct WsView {
   const int32_t* token_sample;   // [T]
   const int32_t* expert_bin;     // [E]
   const int32_t* expert_slot;    // [E]
-  const int32_t* piece_base;     // [n_groups+1] first piece of each 32-token group
+  const int32_t* piece_base;     // [n_groups+1] first piece of each 128-token tile
   const int32_t* sample_pieces;  // [B+1] pieces of sample i are [sp[i], sp[i+1])
   float* pieces;             // [n_pieces * piece_stride]
-  double* mi64;              // [B]
+  float* mi32;               // [B] per-sample MI for the loss
   float* tabs;               // [B * 3 * K]: a_k, b_k, h_k per sample (backward coefficients)
   float* gsave;              // [T * E] softmax scores saved by the forward
   float* dw_part;            // [G * E * d] per-token-group partial dW
+  uint8_t* dz_img;           // [ceil(T/64)][hi|lo][E_pad/64][64 rows][128 B] dz in the MMA layout
   int32_t* perm_scratch;     // permutation block counts / offsets
   uint32_t* attn_ticket;     // [B * ceil(S/128)] head tickets of the attention score
   float* attn_part;          // [H_max * T] per-head vision mass
@@ -51,7 +52,7 @@ struct WsView {
 struct Dims {
   int T, d, E, k, K, B, N_B, renorm;
   int pstride;               // piece_stride(K)
-  int n_groups;              // ceil(T / 32)
+  int n_groups;              // ceil(T / 128): forward tiles = partial-sum groups
 };
 
 struct FwdParams {
@@ -110,6 +111,7 @@ struct PermParams {
   int32_t* blk_offsets;      // [n_blocks * K]
   uint32_t* status;
   int n_blocks;
+  int rounds;                // 256-token rounds per block
 };
 
 struct GaussParams {
@@ -150,6 +152,7 @@ cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX,
                                    const CUtensorMap& tmW, const CUtensorMap& tmDX,
                                    cudaStream_t s);
 cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s);
+cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s);
 cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s);
 cudaError_t launch_gauss_score(const GaussParams& p, smoes_dtype dt, int n_sms, cudaStream_t s);

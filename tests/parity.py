@@ -5,7 +5,12 @@ oracle on the same inputs, and compare with the tolerances the build commits to:
     on tokens whose oracle top-(k+1) logits have no adjacent gap below 1e-3 (near ties can
     legitimately order differently at fp32 accumulation); the excluded count is returned;
   * tensors: ||gpu - ref||_2 <= 2e-3 ||ref||_2 and max|gpu - ref| <= 2e-3 max|ref|;
-  * scalars (MI per sample, loss): |gpu - ref| <= 2e-3 |ref| + 1e-9 nats.
+  * scalars (MI per sample, loss): |gpu - ref| <= 2e-3 |ref| + 1e-9 nats;
+  * outputs stored in bf16 (dX of a bf16 layer): the storage format alone has unit roundoff
+    2^-8 (3.9e-3), above the 2e-3 bar, so each element must lie within one bf16 ulp of the exact
+    oracle value (the correctly rounded value, or its neighbour when the fp32 result sits near a
+    rounding boundary) plus 1e-4 max|ref| for the fp32 accumulation of elements that cancel to
+    near zero, and the norm bar is 2e-3 + 2^-8.
 """
 from __future__ import annotations
 
@@ -46,6 +51,27 @@ def assert_scalar_close(gpu, ref, what):
     assert not np.any(bad), f"{what}: {gpu[bad][:5]} vs {ref[bad][:5]}"
 
 
+def bf16_ulp(x):
+    """Spacing of bf16 numbers at |x| (8 significant bits)."""
+    a = np.abs(np.asarray(x, np.float64))
+    e = np.floor(np.log2(np.where(a > 0, a, 1e-38)))
+    return np.where(a > 0, np.exp2(e - 7), 2.0 ** -133)
+
+
+def assert_bf16_close(gpu, ref, what):
+    gpu = np.asarray(gpu, np.float64)
+    ref = np.asarray(ref, np.float64)
+    assert np.all(np.isfinite(gpu)), f"{what}: non-finite values"
+    err = np.abs(gpu - ref)
+    floor = 1e-4 * (np.abs(ref).max() if ref.size else 0.0)
+    bad = err > bf16_ulp(ref) + floor
+    assert not np.any(bad), (f"{what}: {int(bad.sum())} elements beyond one bf16 ulp; worst "
+                             f"err {err[bad].max():.3e} at |ref| {np.abs(ref[bad]).max():.3e}")
+    r = rel_err(gpu, ref)
+    assert r <= REL + 2.0 ** -8, f"{what}: rel L2 error {r:.3e}"
+    return r
+
+
 def tie_free_tokens(z, k):
     """Tokens whose top-(k+1) logits (fp64 oracle) have all adjacent gaps >= TIE_GAP."""
     kk = min(k + 1, z.shape[1])
@@ -53,6 +79,18 @@ def tie_free_tokens(z, k):
     if kk < 2:
         return np.ones(z.shape[0], bool)
     return np.all(top[:, :-1] - top[:, 1:] >= TIE_GAP, axis=1)
+
+
+def assert_valid_topk(idx, z, k):
+    """For near-tie tokens: the chosen experts are distinct, each is a top-k choice within the
+    tie gap, and they are listed in descending logit order within the tie gap."""
+    if idx.shape[0] == 0:
+        return
+    assert np.all(np.sort(idx, axis=1)[:, 1:] != np.sort(idx, axis=1)[:, :-1]), "repeated expert"
+    kth = -np.sort(-z, axis=1)[:, k - 1]
+    chosen = np.take_along_axis(z, idx.astype(np.int64), axis=1)
+    assert np.all(chosen >= kth[:, None] - TIE_GAP), "an expert outside the top-k was chosen"
+    assert np.all(chosen[:, :-1] >= chosen[:, 1:] - TIE_GAP), "top-k not in descending order"
 
 
 def to_dev(wl, dev):
@@ -120,6 +158,7 @@ def compare(wl, g, ref, check_dx=True):
     ok = tie_free_tokens(fwd["z"], wl.k)
     res["tie_excluded"] = int((~ok).sum())
     np.testing.assert_array_equal(g["topk_idx"][ok], fwd["topk_idx"][ok], err_msg="topk_idx")
+    assert_valid_topk(g["topk_idx"][~ok], fwd["z"][~ok], wl.k)
     res["topk_w"] = assert_tensor_close(g["topk_w"][ok], fwd["topk_w"][ok], "topk_w")
     res["bin_prob"] = assert_tensor_close(g["bin_prob"], fwd["p"], "bin_prob")
     res["joint"] = assert_tensor_close(g["joint"][:wl.B], fwd["joint"], "joint")
@@ -128,7 +167,10 @@ def compare(wl, g, ref, check_dx=True):
     res["dlogits"] = assert_tensor_close(g["dlogits"], ref["dz"], "dlogits")
     res["dW"] = assert_tensor_close(g["dW"], ref["dW"], "dW")
     if check_dx and g["dX"] is not None:
-        res["dX"] = assert_tensor_close(g["dX"], ref["dX"], "dX")
+        if wl.dtype == torch.bfloat16:
+            res["dX"] = assert_bf16_close(g["dX"], ref["dX"], "dX")
+        else:
+            res["dX"] = assert_tensor_close(g["dX"], ref["dX"], "dX")
     # permutation, stage-wise: the oracle permutes the GPU's own top-k, bit for bit
     pr = O.bin_permute(g["topk_idx"], wl.expert_bin, wl.n_bins, is_vision=wl.is_vision)
     np.testing.assert_array_equal(g["offsets"], pr["offsets"], err_msg="bin_offsets")
