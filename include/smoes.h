@@ -183,6 +183,26 @@ smoes_status smoes_bin_permute(smoes_plan plan, const int32_t* topk_idx, const i
                                int32_t* expert_counts, void* ws, size_t ws_bytes,
                                cudaStream_t stream);
 
+/* (4b) The bin permutation of (4) without a workspace, for callers that cannot allocate device
+ *   memory. The paper has no counterpart; this is a deployment convenience. Some callers cannot
+ *   call cudaMalloc: code that runs while a CUDA graph is being captured or that must not trigger
+ *   the implicit device synchronisation cudaMalloc can cause, serving runtimes whose device memory
+ *   is planned up front by an arena that hands out no further blocks, and plug-ins that receive
+ *   only their input and output buffers from a host framework.
+ *   Same arguments and results as smoes_bin_permute, minus the workspace. The scratch it needs
+ *   (about 258 KB: block counts and offsets for up to 1024 permutation blocks x 32 bins, the bin
+ *   map of up to 256 experts, a status word) is a fixed array inside the library, one per device
+ *   that loads it, held until the process exits; this covers every plan smoes_plan_create
+ *   accepts, and larger shapes return SMOES_ERR_UNSUPPORTED.
+ *   The first call on a device looks up that array's device address (once per device); make that
+ *   first call before any stream capture. Every call shares the one array (each call rewrites
+ *   what it reads), so calls that overlap on the GPU, on any stream, race: order them. Device-side
+ *   data errors are recorded in the array's status word only, not reported. */
+smoes_status smoes_bin_permute_noalloc(smoes_plan plan, const int32_t* topk_idx, const int32_t* home,
+                                       const uint8_t* is_vision, int32_t* bin_offsets,
+                                       int32_t* perm_token, uint32_t* perm_mask, int32_t* dispatch,
+                                       int32_t* expert_counts, cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -69,6 +69,7 @@ _sig = {
                               _vp, _vp, _vp, _sz, _vp]),
     "smoes_router_bwd": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _f, _vp, _i, _vp, _vp, _vp, _sz, _vp]),
     "smoes_bin_permute": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "smoes_bin_permute_noalloc": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
 }
 for _name, (_res, _args) in _sig.items():
     _fn = getattr(_lib, _name)
@@ -171,6 +172,15 @@ def smoes_bin_permute(plan, topk_idx, home, is_vision, bin_offsets, perm_token, 
     return _lib.smoes_bin_permute(plan, _p(topk_idx), _p(home), _p(is_vision), _p(bin_offsets),
                                   _p(perm_token), _p(perm_mask), _p(dispatch), _p(expert_counts),
                                   _p(ws), ws.numel() * ws.element_size(), _stream(stream))
+
+
+def smoes_bin_permute_noalloc(plan, topk_idx, home, is_vision, bin_offsets, perm_token, perm_mask,
+                              dispatch, expert_counts, stream=None) -> int:
+    """The permutation without a workspace (scratch inside the library), for callers that cannot
+    allocate device memory; see include/smoes.h for its limits and sharing rules."""
+    return _lib.smoes_bin_permute_noalloc(plan, _p(topk_idx), _p(home), _p(is_vision),
+                                          _p(bin_offsets), _p(perm_token), _p(perm_mask),
+                                          _p(dispatch), _p(expert_counts), _stream(stream))
 
 
 # ----------------------------------------------------------------------------- convenience

@@ -521,3 +521,55 @@ smoes_status smoes_bin_permute(smoes_plan P, const int32_t* topk_idx, const int3
 }
 
 }  // extern "C"
+
+extern "C" smoes_status smoes_bin_permute_noalloc(smoes_plan P, const int32_t* topk_idx,
+                                                  const int32_t* home, const uint8_t* is_vision,
+                                                  int32_t* bin_offsets, int32_t* perm_token,
+                                                  uint32_t* perm_mask, int32_t* dispatch,
+                                                  int32_t* expert_counts, cudaStream_t stream) {
+  if (!P) return SMOES_ERR_INVALID_ARG;
+  const smoes_router_desc& d = P->desc;
+  if (!bin_offsets || !dispatch) return SMOES_ERR_INVALID_ARG;
+  if (expert_counts && !is_vision) return SMOES_ERR_INVALID_ARG;
+  if (P->perm_nblocks > kStaticPermBlocks || d.n_bins > kMaxBins || d.E > kMaxExperts)
+    return SMOES_ERR_UNSUPPORTED;                  // beyond the fixed scratch
+  if (d.T == 0) {
+    cudaError_t e = cudaMemsetAsync(bin_offsets, 0, sizeof(int32_t) * (d.n_bins + 1), stream);
+    if (e == cudaSuccess) e = cudaMemsetAsync(dispatch, 0, sizeof(int32_t) * d.n_bins * d.n_bins, stream);
+    if (e == cudaSuccess && expert_counts) e = cudaMemsetAsync(expert_counts, 0, sizeof(int32_t) * 2 * d.E, stream);
+    return cuda_status(e);
+  }
+  if (!topk_idx || !perm_token || !perm_mask) return SMOES_ERR_INVALID_ARG;
+  StaticPermScratch* sp = nullptr;
+  cudaError_t e = static_perm_scratch(&sp);
+  if (e != cudaSuccess) return SMOES_ERR_CUDA;
+  // the plan's bin map and slots into the scratch; the status word starts at zero
+  e = cudaMemcpyAsync(sp->expert_bin, P->expert_bin.data(), sizeof(int32_t) * d.E,
+                      cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(sp->expert_slot, P->expert_slot.data(), sizeof(int32_t) * d.E,
+                        cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(sp->status, 0, sizeof(sp->status), stream);
+  if (e != cudaSuccess) return SMOES_ERR_CUDA;
+  PermParams p{};
+  p.T = d.T;
+  p.k = d.k;
+  p.E = d.E;
+  p.K = d.n_bins;
+  p.topk_idx = topk_idx;
+  p.home = home;
+  p.is_vision = is_vision;
+  p.expert_bin = sp->expert_bin;
+  p.expert_slot = sp->expert_slot;
+  p.bin_offsets = bin_offsets;
+  p.perm_token = perm_token;
+  p.perm_mask = perm_mask;
+  p.dispatch = dispatch;
+  p.expert_counts = expert_counts;
+  p.blk_counts = sp->blk_counts;
+  p.blk_offsets = sp->blk_offsets;
+  p.status = sp->status;
+  p.n_blocks = P->perm_nblocks;
+  p.rounds = perm_rounds(d.T);
+  return cuda_status(launch_bin_permute(p, stream));
+}

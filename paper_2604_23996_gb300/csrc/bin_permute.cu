@@ -7,6 +7,8 @@
 //   scan    block offsets per bin and the bin offsets (one block, warp-shuffle scans);
 //   scatter stable positions from ballots + block offsets, writes tokens and masks, and adds the
 //           dispatch matrix and per-modality expert counts (integer atomics: order-independent).
+#include <mutex>
+
 #include "device_common.cuh"
 #include "smoes_internal.cuh"
 
@@ -183,6 +185,31 @@ __global__ void __launch_bounds__(kPermThreads) k_perm_scatter(const PermParams 
 }
 
 }  // namespace
+
+// Scratch of the no-allocation permutation entry point (see smoes_bin_permute_noalloc): one copy
+// per device that loads this library, alive until the process exits, shared by every call.
+static __device__ __align__(256) unsigned char g_perm_static[sizeof(StaticPermScratch)];
+
+// The host cannot use g_perm_static's name as a device address; it asks the runtime once per
+// device, with that device current, and caches the answer.
+cudaError_t static_perm_scratch(StaticPermScratch** out) {
+  constexpr int kMaxDevices = 64;
+  static std::mutex mu;
+  static void* addr[kMaxDevices] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_perm_static);
+    if (e != cudaSuccess) return e;
+    addr[dev] = p;
+  }
+  *out = static_cast<StaticPermScratch*>(addr[dev]);
+  return cudaSuccess;
+}
 
 // Rounds of 256 tokens per block: 1 while that keeps the block count <= 1024 (the scan runs in
 // one block of 1024 threads), more for larger batches.

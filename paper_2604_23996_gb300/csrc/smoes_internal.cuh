@@ -144,6 +144,20 @@ struct AttnParams {
   uint64_t limit_ns;
 };
 
+// Fixed-size scratch of smoes_bin_permute_noalloc, kept in a file-scope __device__ array of
+// bin_permute.cu (for callers that cannot allocate): room for 1024 permutation blocks x 32 bins
+// and 256 experts, which covers every plan smoes_plan_create accepts.
+constexpr int kStaticPermBlocks = 1024;
+struct StaticPermScratch {
+  int32_t blk_counts[kStaticPermBlocks * kMaxBins];
+  int32_t blk_offsets[kStaticPermBlocks * kMaxBins];
+  int32_t expert_bin[kMaxExperts];
+  int32_t expert_slot[kMaxExperts];
+  uint32_t status[4];
+};
+// Device address of that array on the current device (resolved once per device).
+cudaError_t static_perm_scratch(StaticPermScratch** out);
+
 // ------------------------------------------------------------------ launchers (in .cu files)
 cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
                                    const CUtensorMap& tmW, int n_sms, cudaStream_t s);
