@@ -22,28 +22,49 @@ __global__ void __launch_bounds__(256) k_gauss_score(const GaussParams p) {
   const float gc = gauss_coefficients(p.mu, p.var, p.d, dpad, ga, gb, red, p.status);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int per = kBf16 ? 8 : 4;                      // elements per 16-byte load
+  constexpr int kU = 4;                               // 16-byte loads in flight per lane
   for (int j = blockIdx.x * 8 + warp; j < p.T; j += gridDim.x * 8) {
     float acc = 0.f;
     if (kBf16) {
       const __nv_bfloat16* row = static_cast<const __nv_bfloat16*>(p.X) + static_cast<size_t>(j) * p.d;
-      for (int c = lane * per; c < p.d; c += 32 * per) {
-        const uint4 u = __ldg(reinterpret_cast<const uint4*>(row + c));
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+      for (int c0 = lane * per; c0 < p.d; c0 += 32 * per * kU) {
+        uint4 u[kU];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          const float x0 = __uint_as_float(w[q] << 16), x1 = __uint_as_float(w[q] & 0xffff0000u);
-          acc = fmaf(x0, fmaf(ga[c + 2 * q], x0, gb[c + 2 * q]), acc);
-          acc = fmaf(x1, fmaf(ga[c + 2 * q + 1], x1, gb[c + 2 * q + 1]), acc);
+        for (int q = 0; q < kU; ++q) {
+          const int c = c0 + q * 32 * per;
+          u[q] = c < p.d ? __ldg(reinterpret_cast<const uint4*>(row + c)) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int q = 0; q < kU; ++q) {
+          const int c = c0 + q * 32 * per;
+          if (c >= p.d) break;
+          const uint32_t w[4] = {u[q].x, u[q].y, u[q].z, u[q].w};
+#pragma unroll
+          for (int r = 0; r < 4; ++r) {
+            const float x0 = __uint_as_float(w[r] << 16), x1 = __uint_as_float(w[r] & 0xffff0000u);
+            acc = fmaf(x0, fmaf(ga[c + 2 * r], x0, gb[c + 2 * r]), acc);
+            acc = fmaf(x1, fmaf(ga[c + 2 * r + 1], x1, gb[c + 2 * r + 1]), acc);
+          }
         }
       }
     } else {
       const float* row = static_cast<const float*>(p.X) + static_cast<size_t>(j) * p.d;
-      for (int c = lane * per; c < p.d; c += 32 * per) {
-        const float4 u = __ldg(reinterpret_cast<const float4*>(row + c));
-        acc = fmaf(u.x, fmaf(ga[c], u.x, gb[c]), acc);
-        acc = fmaf(u.y, fmaf(ga[c + 1], u.y, gb[c + 1]), acc);
-        acc = fmaf(u.z, fmaf(ga[c + 2], u.z, gb[c + 2]), acc);
-        acc = fmaf(u.w, fmaf(ga[c + 3], u.w, gb[c + 3]), acc);
+      for (int c0 = lane * per; c0 < p.d; c0 += 32 * per * kU) {
+        float4 u[kU];
+#pragma unroll
+        for (int q = 0; q < kU; ++q) {
+          const int c = c0 + q * 32 * per;
+          u[q] = c < p.d ? __ldg(reinterpret_cast<const float4*>(row + c)) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int q = 0; q < kU; ++q) {
+          const int c = c0 + q * 32 * per;
+          if (c >= p.d) break;
+          acc = fmaf(u[q].x, fmaf(ga[c], u[q].x, gb[c]), acc);
+          acc = fmaf(u[q].y, fmaf(ga[c + 1], u[q].y, gb[c + 1]), acc);
+          acc = fmaf(u[q].z, fmaf(ga[c + 2], u[q].z, gb[c + 2]), acc);
+          acc = fmaf(u[q].w, fmaf(ga[c + 3], u[q].w, gb[c + 3]), acc);
+        }
       }
     }
     acc = warp_sum(acc);
