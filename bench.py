@@ -237,11 +237,14 @@ def main():
         dist.init_process_group("nccl", device_id=dev)
 
     from paper_2604_23996_gb300 import binding as bd
-    from paper_2604_23996_gb300.workloads import config_workload
+    from paper_2604_23996_gb300.workloads import attn_workload, config_workload
 
     wl = config_workload(args.config)
+    use_attn = args.config == "attn_router"
+    aw = attn_workload() if use_attn else None
     dtype = bd.SMOES_BF16 if wl.dtype == torch.bfloat16 else bd.SMOES_F32
-    r = bd.Router(wl.T, wl.d, wl.E, wl.k, wl.n_bins, wl.sample_offsets, wl.expert_bin, dtype)
+    r = bd.Router(wl.T, wl.d, wl.E, wl.k, wl.n_bins, wl.sample_offsets, wl.expert_bin, dtype,
+                  attn_max_heads=aw.H if use_attn else 0)
     X = wl.X.to(dev)
     W = wl.W.to(dev)
     mu, var = wl.mu.to(dev), wl.var.to(dev)
@@ -249,43 +252,55 @@ def main():
     dW = torch.empty((wl.E, wl.d), dtype=torch.float32, device=dev)
     dX = torch.empty_like(X)
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)   # 256 MiB > L2
+    Ma = torch.empty((wl.T, 2), dtype=torch.float32, device=dev)
+    if use_attn:
+        attn = dict(Q=aw.Q.to(dev), K=aw.K.to(dev), B=aw.B, H=aw.H, S=aw.S, hd=aw.hd,
+                    sm_scale=aw.sm_scale, causal=1, key_bias=torch.from_numpy(aw.key_bias).to(dev),
+                    is_vision=torch.from_numpy(aw.is_vision).to(dev))
+
+    def score():
+        r.modality_score(bd.SMOES_SCORE_ATTN, Ma, attn=attn)
 
     def fwd():
-        r.forward(X, W, mu=mu, var=var, tau=wl.tau, bin_prob=False)
+        if use_attn:
+            r.forward(X, W, M_in=Ma, bin_prob=False)
+        else:
+            r.forward(X, W, mu=mu, var=var, tau=wl.tau, bin_prob=False)
 
     def bwd():
-        r.backward(X, W, r.M, dW, dX=dX, loss_scale=1e-4)
+        r.backward(X, W, Ma if use_attn else r.M, dW, dX=dX, loss_scale=1e-4)
 
     def perm():
         r.permute(is_vision=is_vis)
 
+    parts = ([("attn", score)] if use_attn else []) + [("fwd", fwd), ("bwd", bwd), ("permute", perm)]
+
     # eager warm-up (also checks the device status once), then graph capture per call
     for _ in range(2):
-        fwd(); bwd(); perm()
+        for _, fn in parts:
+            fn()
     code, _ = r.device_status()
     assert code == 0, f"device status {code}"
     graphs = []
     s = torch.cuda.Stream(device=dev)
     s.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(s):
-        for fn in (fwd, bwd, perm):
+        for _, fn in parts:
             g = torch.cuda.CUDAGraph()
             with torch.cuda.graph(g, stream=s):
                 fn()
             graphs.append(g)
     torch.cuda.current_stream().wait_stream(s)
     torch.cuda.synchronize()
-    launches_per_step = 6          # fwd 1, bwd 2 (main + dW reduce), permutation 3
+    # our kernels per step: attention 1, fwd 1, bwd 3 (dz prep, main, dW reduce), permutation 3
+    launches_per_step = (1 if use_attn else 0) + 1 + (3 if dtype == bd.SMOES_BF16 else 2) + 3
 
     def step_timed():
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(parts) + 1)]
         ev[0].record()
-        graphs[0].replay()
-        ev[1].record()
-        graphs[1].replay()
-        ev[2].record()
-        graphs[2].replay()
-        ev[3].record()
+        for i, g in enumerate(graphs):
+            g.replay()
+            ev[i + 1].record()
         return ev
 
     for _ in range(args.warmup):
@@ -316,10 +331,9 @@ def main():
         dist.barrier()
     torch.cuda.synchronize()
     clk = clocks.stop() if not args.profile else {"sm_mhz": None, "note": "profile run"}
-    t_step = [e[0].elapsed_time(e[3]) for e in evs]
-    t_fwd = [e[0].elapsed_time(e[1]) for e in evs]
-    t_bwd = [e[1].elapsed_time(e[2]) for e in evs]
-    t_perm = [e[2].elapsed_time(e[3]) for e in evs]
+    t_step = [e[0].elapsed_time(e[-1]) for e in evs]
+    t_part = {name: [e[i].elapsed_time(e[i + 1]) for e in evs] for i, (name, _) in enumerate(parts)}
+    t_bwd = t_part["bwd"]
     total_ms = float(np.sum(t_step))
     if world > 1:
         t = torch.tensor([total_ms], device=dev)
@@ -339,12 +353,20 @@ def main():
                muh.numel() * 4 + varh.numel() * 4)
         d2h = 4
 
+        if use_attn:
+            Qh, Kh = aw.Q.pin_memory(), aw.K.pin_memory()
+            h2d += 2 * Qh.numel() * Qh.element_size()
+
         def e2e_step():
             X.copy_(Xh, non_blocking=True)
             W.copy_(Wh, non_blocking=True)
             mu.copy_(muh, non_blocking=True)
             var.copy_(varh, non_blocking=True)
-            fwd(); bwd(); perm()
+            if use_attn:
+                attn["Q"].copy_(Qh, non_blocking=True)
+                attn["K"].copy_(Kh, non_blocking=True)
+            for _, fn in parts:
+                fn()
             lossh.copy_(r.loss, non_blocking=True)
 
         for _ in range(3):
@@ -370,17 +392,25 @@ def main():
 
     hbm, tf_burst, tf_sus, peak_kind = peaks()
     step_bytes, step_flops, bwd_bytes, bwd_flops = algorithmic(wl)
+    if use_attn:   # causal Q K^T of the attention score: B H S^2 hd flops; Q and K read once
+        attn_flops = float(aw.B) * aw.H * aw.S * aw.S * aw.hd
+        attn_bytes = 2.0 * aw.Q.numel() * aw.Q.element_size()
+    else:
+        attn_flops = attn_bytes = 0.0
     bwd_ms = float(np.mean(t_bwd))
     achieved = bwd_bytes / (bwd_ms * 1e-3) / 1e9
-    t_roof = max(step_bytes / (hbm * 1e9), step_flops / (tf_sus * 1e12))
+    t_roof = (max(step_bytes / (hbm * 1e9), step_flops / (tf_sus * 1e12)) +
+              max(attn_bytes / (hbm * 1e9), attn_flops / (tf_sus * 1e12)))
     traffic = profile_traffic("router_bwd.cu", args.config)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == torch.bfloat16 else "f32",
         "data": "synthetic (seeded; shapes of the paper's MoE-VLM router layers)",
-        "config": {"workload": f"{args.config}: {WORKLOAD_TEXT[args.config]}; Gaussian score; "
-                               "fwd + bwd (dW, dX) + bin permutation",
+        "config": {"workload": f"{args.config}: {WORKLOAD_TEXT[args.config]}; "
+                               + ("attention score (8x4096, 16 heads, hd 128, causal) + " if use_attn
+                                  else "Gaussian score; ")
+                               + "fwd + bwd (dW, dX) + bin permutation",
                    "l2": "flushed before every step (256 MiB write, outside the timed interval)",
                    "clocks": "nvidia-smi every 100 ms over a load window of ~0.5 s of steps "
                              "ending with the timed steps",
@@ -391,9 +421,8 @@ def main():
                      "peak_source": peak_kind},
         "step_roofline": {"t_roof_us": t_roof * 1e6, "t_step_us": ms_per_step * 1e3,
                           "frac": t_roof / (ms_per_step * 1e-3),
-                          "bytes": step_bytes, "flops": step_flops},
-        "breakdown_us": {"fwd": 1e3 * float(np.mean(t_fwd)), "bwd": 1e3 * bwd_ms,
-                         "permute": 1e3 * float(np.mean(t_perm))},
+                          "bytes": step_bytes + attn_bytes, "flops": step_flops + attn_flops},
+        "breakdown_us": {name: 1e3 * float(np.mean(v)) for name, v in t_part.items()},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
         "e2e": e2e,

@@ -50,7 +50,8 @@ __device__ __forceinline__ void topk_push(uint32_t (&tk)[KM], uint32_t q) {
 // eps_mk = N_mk n / (Q_k A_m) - 1. With s_m = sum_k q_k eps_mk (so N_B sum_k Sbar_mk = 1 + s_m),
 //   P_mk = q_k (1 + eps_mk) / (2 + s_v + s_t),
 //   log(P_mk / (P_m P_k)) = log1p(eps_mk) - log1p((eps_vk + eps_tk)/2) + log1p((s_v + s_t)/2) - log1p(s_m),
-// every term a log1p of a small, directly computed quantity.
+// every term a log1p of a small, directly computed quantity; h_k is formed from second-order
+// differences directly as well (see below).
 constexpr int kReduceRound = 16;             // pieces loaded per round before they are summed
 
 __device__ void sample_reduce(const FwdParams& p, int s) {
@@ -122,7 +123,7 @@ __device__ void sample_reduce(const FwdParams& p, int s) {
   }
   const float sv = warp_sum(q * ev), st = warp_sum(q * et);
   const float NB = static_cast<float>(dm.N_B);
-  float Pv = 0.f, Pt = 0.f, a = 0.f, b = 0.f, I = 0.f;
+  float Pv = 0.f, Pt = 0.f, a = 0.f, b = 0.f, h = 0.f, I = 0.f;
   if (has_v && has_t) {
     const float nbz = 2.f + sv + st;                               // N_B * Z
     Pv = q * (1.f + ev) / nbz;                                     // eq. (13)
@@ -134,6 +135,19 @@ __device__ void sample_reduce(const FwdParams& p, int s) {
     const float Z = nbz / NB;
     a = act ? (Lv - I) / Z / (NB * Av) : 0.f;
     b = act ? (Lt - I) / Z / (NB * At) : 0.f;
+    if (cv && ct && act) {
+      // h = (a + b) / 2 is second order (a ~ -b): form L_v + L_t and 1/A_v - 1/A_t directly,
+      //   L_v + L_t = log1p(-(d/(1+m))^2) - log1p(-(d_s/(1+m_s))^2),
+      // with m, d the half-sum and half-difference of (eps_v, eps_t) and m_s, d_s those of (s_v, s_t).
+      const float yv = 2.f * Dv / n, yt = 2.f * Dt / n;
+      const float m = 0.5f * (ev + et), dd = 0.5f * (ev - et);
+      const float ms = 0.5f * (sv + st), ds = 0.5f * (sv - st);
+      const float rk = dd / (1.f + m), rs = ds / (1.f + ms);
+      const float S2 = log1pf(-rk * rk) - log1pf(-rs * rs);
+      h = ((S2 - 2.f * I) / (1.f + yv) + (Lt - I) * (yv - yt) / ((1.f + yv) * (1.f + yt))) / (Z * NB * n);
+    } else {
+      h = 0.5f * (a + b);
+    }
   } else if (has_v || has_t) {                                     // one modality only: I = 0
     const float e1 = has_v ? ev : et, s1 = has_v ? sv : st;
     const float P1 = q * (1.f + e1) / (1.f + s1);
@@ -144,7 +158,7 @@ __device__ void sample_reduce(const FwdParams& p, int s) {
     float* tb = p.ws.tabs + static_cast<size_t>(s) * 3 * K;
     tb[lane] = a;
     tb[K + lane] = b;
-    tb[2 * K + lane] = 0.5f * (a + b);
+    tb[2 * K + lane] = h;
     if (p.joint) {
       p.joint[(static_cast<size_t>(s) * 2 + 0) * K + lane] = Pv;
       p.joint[(static_cast<size_t>(s) * 2 + 1) * K + lane] = Pt;
