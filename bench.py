@@ -292,8 +292,11 @@ def main():
             graphs.append(g)
     torch.cuda.current_stream().wait_stream(s)
     torch.cuda.synchronize()
-    # our kernels per step: attention 1, fwd 1, bwd 3 (dz prep, main, dW reduce), permutation 3
-    launches_per_step = (1 if use_attn else 0) + 1 + (3 if dtype == bd.SMOES_BF16 else 2) + 3
+    # our kernels per step: attention 1, fwd 1 (+1 Gaussian coefficients on the fp32 path),
+    # bwd 3 (dz prep, main, dW reduce; fp32: main, dW reduce), permutation 1
+    f32 = dtype != bd.SMOES_BF16
+    launches_per_step = ((1 if use_attn else 0) + 1 + (1 if f32 and not use_attn else 0)
+                         + (2 if f32 else 3) + 1)
 
     def step_timed():
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(parts) + 1)]

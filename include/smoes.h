@@ -190,7 +190,7 @@ smoes_status smoes_bin_permute(smoes_plan plan, const int32_t* topk_idx, const i
  *   is planned up front by an arena that hands out no further blocks, and plug-ins that receive
  *   only their input and output buffers from a host framework.
  *   Same arguments and results as smoes_bin_permute, minus the workspace. The scratch it needs
- *   (about 258 KB: block counts and offsets for up to 1024 permutation blocks x 32 bins, the bin
+ *   (about 130 KB: block counts for up to 1024 permutation blocks x 32 bins, the bin
  *   map of up to 256 experts, a status word) is a fixed array inside the library, one per device
  *   that loads it, held until the process exits; this covers every plan smoes_plan_create
  *   accepts, and larger shapes return SMOES_ERR_UNSUPPORTED.

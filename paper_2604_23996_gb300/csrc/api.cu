@@ -23,7 +23,8 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
   size_t status, sample_ticket, loss_ticket, offsets, token_sample, expert_bin, expert_slot,
-      piece_base, sample_pieces, pieces, mi32, tabs, gsave, dw_part, dz_img, perm, attn_ticket, attn_part;
+      piece_base, sample_pieces, pieces, mi32, tabs, gsave, dw_part, dz_img, perm, attn_ticket, attn_part,
+      gcoef, perm_sync;
   size_t header_bytes;   // [0, header_bytes) is cleared by smoes_workspace_init
   size_t total;
 };
@@ -40,6 +41,8 @@ struct smoes_plan_s {
   int bwd_tiles = 0;     // 64-token tiles
   int bwd_groups = 1, bwd_slices = 1, bwd_slice_width = 0;
   int perm_nblocks = 0;
+  int dcoef = 256;       // Gaussian coefficient vectors padded to 256 features
+  bool contig_bins = false;
   std::vector<int32_t> offsets, expert_bin, expert_slot, token_sample, piece_base, sample_pieces;
   Layout L{};
 };
@@ -70,6 +73,8 @@ WsView make_view(const smoes_plan_s* P, void* ws) {
   v.perm_scratch = reinterpret_cast<int32_t*>(b + L.perm);
   v.attn_ticket = reinterpret_cast<uint32_t*>(b + L.attn_ticket);
   v.attn_part = reinterpret_cast<float*>(b + L.attn_part);
+  v.gcoef = reinterpret_cast<float*>(b + L.gcoef);
+  v.dcoef = P->dcoef;
   return v;
 }
 
@@ -86,6 +91,7 @@ Dims make_dims(const smoes_plan_s* P) {
   m.renorm = d.renorm_topk ? 1 : 0;
   m.pstride = piece_stride(d.n_bins);
   m.n_groups = P->n_groups;
+  m.contig_bins = P->contig_bins ? 1 : 0;
   return m;
 }
 
@@ -119,6 +125,21 @@ bool encode_bf16_2d(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t col
   const cuuint32_t box[2] = {box_cols, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE,
+             swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// 2-D row-major fp32 tensor [rows, cols] (cols * 4 a multiple of 16); box [box_rows, box_cols].
+bool encode_f32_2d(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                   uint32_t box_cols, bool swizzle128) {
+  EncodeTiledFn enc = get_encode();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {cols * 4};
+  const cuuint32_t box[2] = {box_cols, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(ptr), dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE,
              swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -200,6 +221,10 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   }
   for (int b = 0; b < K; ++b)
     if (fill[b] != P->N_B) { delete P; return SMOES_ERR_INVALID_ARG; }
+  // consecutive bins of a multiple of 4 experts: the forward sums bins in 4-expert groups
+  P->contig_bins = P->N_B % 4 == 0;
+  for (int e = 0; e < E && P->contig_bins; ++e) P->contig_bins = P->expert_bin[e] == e / P->N_B;
+  P->dcoef = round_up(d.d, 256);
 
   // token -> sample, 32-token groups -> pieces (one piece per (group, sample) pair)
   P->n_groups = (T + kPieceTokens - 1) / kPieceTokens;
@@ -246,6 +271,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.sample_ticket = take(sizeof(uint32_t) * std::max(B, 1));
   L.loss_ticket = take(sizeof(uint32_t) * 4);
   L.attn_ticket = take(sizeof(uint32_t) * (static_cast<size_t>(T) + 1));
+  L.perm_sync = take(sizeof(uint32_t) * 4);
   L.header_bytes = o;
   L.offsets = take(sizeof(int32_t) * (B + 1));
   L.token_sample = take(sizeof(int32_t) * std::max(T, 1));
@@ -260,8 +286,9 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.dw_part = take(sizeof(float) * static_cast<size_t>(P->bwd_groups) * E * d.d);
   L.dz_img = take(d.dtype == SMOES_BF16 && E <= 128
                       ? static_cast<size_t>(P->bwd_tiles) * 2 * round_up(E, 64) * 128 : 0);
-  L.perm = take(sizeof(int32_t) * 2 * static_cast<size_t>(P->perm_nblocks) * K);
+  L.perm = take(sizeof(int32_t) * static_cast<size_t>(P->perm_nblocks) * K);
   L.attn_part = take(sizeof(float) * static_cast<size_t>(T) * std::max(0, d.attn_max_heads));
+  L.gcoef = take(sizeof(float) * (2 * static_cast<size_t>(P->dcoef) + P->dcoef / 256));
   L.total = o;
   *out = P;
   return SMOES_OK;
@@ -324,12 +351,14 @@ smoes_status smoes_modality_score(smoes_plan P, smoes_score_mode mode, const smo
     p.T = d.T;
     p.d = d.d;
     p.X = g.X;
-    p.mu = g.mu;
-    p.var = g.var;
+    p.gcoef = v.gcoef;
+    p.dcoef = v.dcoef;
     p.inv_tau = 1.f / (g.tau > 0.f ? g.tau : 0.5f * d.d);
     p.M = M;
     p.status = v.status;
-    return cuda_status(launch_gauss_score(p, d.dtype, P->n_sms, stream));
+    cudaError_t e = launch_gauss_coef(g.mu, g.var, d.d, v.dcoef, v.gcoef, v.status, stream);
+    if (e == cudaSuccess) e = launch_gauss_score(p, d.dtype, P->n_sms, stream);
+    return cuda_status(e);
   }
   if (mode == SMOES_SCORE_ATTN) {
     const smoes_attn_args& a = args->attn;
@@ -387,7 +416,8 @@ smoes_status smoes_router_fwd(smoes_plan P, const void* X, const void* W, const 
   if (!X || !W || !topk_idx || !topk_w || !mi) return SMOES_ERR_INVALID_ARG;
   if ((M_in == nullptr) == (gauss == nullptr)) return SMOES_ERR_INVALID_ARG;
   if (gauss && (!gauss->mu || !gauss->var || !M_out)) return SMOES_ERR_INVALID_ARG;
-  if (!aligned16(X) || !aligned16(W) || (M_in && !aligned16(M_in)) || (M_out && !aligned16(M_out)))
+  if (!aligned16(X) || !aligned16(W) || (M_in && !aligned16(M_in)) || (M_out && !aligned16(M_out)) ||
+      (gauss && (!aligned16(gauss->mu) || !aligned16(gauss->var))))
     return SMOES_ERR_ALIGNMENT;
   if (d.dtype == SMOES_F32 && d.E > 64) return SMOES_ERR_UNSUPPORTED;
 
@@ -408,13 +438,21 @@ smoes_status smoes_router_fwd(smoes_plan P, const void* X, const void* W, const 
   p.mi = mi;
   p.loss = loss;
   p.limit_ns = kWaitLimitNs;
+  if (gauss && d.dtype == SMOES_F32) {
+    const cudaError_t e = launch_gauss_coef(gauss->mu, gauss->var, d.d, p.ws.dcoef, p.ws.gcoef,
+                                            p.ws.status, stream);
+    if (e != cudaSuccess) return SMOES_ERR_CUDA;
+  }
   if (d.dtype == SMOES_BF16) {
     p.n_tiles = (d.T + kFwdBM - 1) / kFwdBM;
     CUtensorMap tx, tw;
     if (!encode_bf16_2d(&tx, X, d.T, d.d, kFwdBM, kFwdBK, true) ||
         !encode_bf16_2d(&tw, W, d.E, d.d, round_up(d.E, 16), kFwdBK, true))
       return SMOES_ERR_CUDA;
-    return cuda_status(launch_router_fwd_bf16(p, tx, tw, P->n_sms, stream));
+    // saved scores leave through TMA when their rows are 16-byte multiples
+    CUtensorMap tg;
+    const bool tma_g = d.E % 4 == 0 && d.E <= 128 && encode_f32_2d(&tg, p.ws.gsave, d.T, d.E, 128, 32, true);
+    return cuda_status(launch_router_fwd_bf16(p, tx, tw, tma_g ? &tg : nullptr, P->n_sms, stream));
   }
   p.n_tiles = P->n_groups;
   return cuda_status(launch_router_fwd_f32(p, stream));
@@ -513,10 +551,11 @@ smoes_status smoes_bin_permute(smoes_plan P, const int32_t* topk_idx, const int3
   p.dispatch = dispatch;
   p.expert_counts = expert_counts;
   p.blk_counts = v.perm_scratch;
-  p.blk_offsets = v.perm_scratch + static_cast<size_t>(P->perm_nblocks) * d.n_bins;
+  p.sync = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + P->L.perm_sync);
   p.status = v.status;
   p.n_blocks = P->perm_nblocks;
   p.rounds = perm_rounds(d.T);
+  p.limit_ns = kWaitLimitNs;
   return cuda_status(launch_bin_permute(p, stream));
 }
 
@@ -543,13 +582,14 @@ extern "C" smoes_status smoes_bin_permute_noalloc(smoes_plan P, const int32_t* t
   StaticPermScratch* sp = nullptr;
   cudaError_t e = static_perm_scratch(&sp);
   if (e != cudaSuccess) return SMOES_ERR_CUDA;
-  // the plan's bin map and slots into the scratch; the status word starts at zero
+  // the plan's bin map and slots into the scratch; the status and barrier words start at zero
   e = cudaMemcpyAsync(sp->expert_bin, P->expert_bin.data(), sizeof(int32_t) * d.E,
                       cudaMemcpyHostToDevice, stream);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(sp->expert_slot, P->expert_slot.data(), sizeof(int32_t) * d.E,
                         cudaMemcpyHostToDevice, stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(sp->status, 0, sizeof(sp->status), stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(sp->sync, 0, sizeof(sp->sync), stream);
   if (e != cudaSuccess) return SMOES_ERR_CUDA;
   PermParams p{};
   p.T = d.T;
@@ -567,9 +607,10 @@ extern "C" smoes_status smoes_bin_permute_noalloc(smoes_plan P, const int32_t* t
   p.dispatch = dispatch;
   p.expert_counts = expert_counts;
   p.blk_counts = sp->blk_counts;
-  p.blk_offsets = sp->blk_offsets;
+  p.sync = sp->sync;
   p.status = sp->status;
   p.n_blocks = P->perm_nblocks;
   p.rounds = perm_rounds(d.T);
+  p.limit_ns = kWaitLimitNs;
   return cuda_status(launch_bin_permute(p, stream));
 }

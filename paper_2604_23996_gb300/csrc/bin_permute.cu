@@ -2,20 +2,24 @@
 //
 // Every token is sent once to each bin that holds at least one of its top-k experts; the
 // entry carries a bit mask of the chosen experts' slots inside the bin. Entries are grouped by
-// bin (ascending) and ordered by token inside a bin. Three launches, all integer work:
-//   count   per-block pair counts per bin (warp ballots), zeroes the atomic outputs;
-//   scan    block offsets per bin and the bin offsets (one block, warp-shuffle scans);
-//   scatter stable positions from ballots + block offsets, writes tokens and masks, and adds the
-//           dispatch matrix and per-modality expert counts (integer atomics: order-independent).
+// bin (ascending) and ordered by token inside a bin. One cooperative launch, all integer work:
+//   count    per-block pair counts per bin (warp ballots);
+//   barrier  a bounded grid barrier (all blocks are resident: cooperative launch);
+//   offsets  each block sums the count table: its prefix inside every bin and the bin bases;
+//   scatter  stable positions from ballots, tokens and masks written, and the dispatch matrix
+//            and per-modality expert counts added (integer atomics: order-independent).
+#include <algorithm>
 #include <mutex>
 
 #include "device_common.cuh"
+#include "ptx.cuh"
 #include "smoes_internal.cuh"
 
 namespace smoes {
 namespace {
 
 constexpr int kPermThreads = 256;                    // one token per thread and round
+constexpr int kPermWarps = kPermThreads / 32;
 
 struct TokenSel {
   int e[kMaxTopK];
@@ -23,17 +27,19 @@ struct TokenSel {
   uint32_t bins;
 };
 
-__device__ __forceinline__ void load_sel(const PermParams& p, int j, TokenSel& s) {
+__device__ __forceinline__ void load_sel(const PermParams& p, const int* s_bin, int j, TokenSel& s) {
   s.bins = 0u;
+  int e[kMaxTopK];
+#pragma unroll
+  for (int i = 0; i < kMaxTopK; ++i) e[i] = i < p.k ? p.topk_idx[static_cast<size_t>(j) * p.k + i] : -1;
 #pragma unroll
   for (int i = 0; i < kMaxTopK; ++i) {
     s.e[i] = -1;
     s.b[i] = -1;
     if (i < p.k) {
-      const int e = p.topk_idx[static_cast<size_t>(j) * p.k + i];
-      if (e >= 0 && e < p.E) {
-        s.e[i] = e;
-        s.b[i] = p.expert_bin[e];
+      if (e[i] >= 0 && e[i] < p.E) {
+        s.e[i] = e[i];
+        s.b[i] = s_bin[e[i]];
         s.bins |= 1u << s.b[i];
       } else {
         atomicOr(p.status, kStatusData);
@@ -42,113 +48,134 @@ __device__ __forceinline__ void load_sel(const PermParams& p, int j, TokenSel& s
   }
 }
 
-__global__ void __launch_bounds__(kPermThreads) k_perm_count(const PermParams p) {
-  __shared__ int wc[kPermThreads / 32][kMaxBins];
+// Grid barrier for co-resident blocks, called by one thread per block. sync[0] counts
+// arrivals, sync[1] is the generation; the last block resets the count and advances the
+// generation, so the pair is zero-count again between calls. A wait that exceeds limit_ns sets
+// the timeout status and returns false.
+__device__ bool grid_barrier(uint32_t* sync, uint32_t n, uint64_t limit_ns, uint32_t* status) {
+  volatile uint32_t* gen = sync + 1;
+  const uint32_t g0 = *gen;
+  __threadfence();
+  if (atomicAdd(sync, 1u) == n - 1) {
+    atomicExch(sync, 0u);
+    __threadfence();
+    atomicAdd(sync + 1, 1u);
+    return true;
+  }
+  const uint64_t t0 = global_ns();
+  while (*gen == g0) {
+    if (global_ns() - t0 > limit_ns) {
+      atomicOr(status, kStatusTimeout);
+      return false;
+    }
+    __nanosleep(64);
+  }
+  __threadfence();
+  return true;
+}
+
+__global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
+  __shared__ int s_bin[kMaxExperts];
+  __shared__ int s_slot[kMaxExperts];
+  __shared__ int wcnt[kPermWarps][kMaxBins];
+  __shared__ int base[kMaxBins];
+  __shared__ int pre_s[kMaxBins], tot_s[kMaxBins];
+  __shared__ int disp[kMaxBins * kMaxBins];
+  __shared__ int ecnt[2 * kMaxExperts];
+  __shared__ int ok_s;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  int cnt = 0;                                          // lane kb of each warp counts bin kb
+  const int K = p.K;
+  for (int e = threadIdx.x; e < p.E; e += kPermThreads) {
+    s_bin[e] = p.expert_bin[e];
+    s_slot[e] = p.expert_slot[e];
+  }
+  for (int i = threadIdx.x; i < K * K; i += kPermThreads) disp[i] = 0;
+  for (int i = threadIdx.x; i < 2 * p.E; i += kPermThreads) ecnt[i] = 0;
+  __syncthreads();
+
+  // count: lane kb of each warp accumulates the warp's pairs in bin kb
+  int cnt = 0;
   for (int r = 0; r < p.rounds; ++r) {
     const int j = (blockIdx.x * p.rounds + r) * kPermThreads + threadIdx.x;
     TokenSel s;
     s.bins = 0u;
-    if (j < p.T) load_sel(p, j, s);
-    for (int kb = 0; kb < p.K; ++kb) {
+    if (j < p.T) load_sel(p, s_bin, j, s);
+    for (int kb = 0; kb < K; ++kb) {
       const int c = __popc(__ballot_sync(0xffffffffu, (s.bins >> kb) & 1u));
       if (lane == kb) cnt += c;
     }
   }
-  if (lane < kMaxBins) wc[warp][lane] = cnt;
+  if (lane < kMaxBins) wcnt[warp][lane] = cnt;
   __syncthreads();
-  if (threadIdx.x < p.K) {
+  if (threadIdx.x < K) {
     int t = 0;
-    for (int w = 0; w < kPermThreads / 32; ++w) t += wc[w][threadIdx.x];
-    p.blk_counts[blockIdx.x * p.K + threadIdx.x] = t;
+    for (int w = 0; w < kPermWarps; ++w) t += wcnt[w][threadIdx.x];
+    p.blk_counts[blockIdx.x * K + threadIdx.x] = t;
   }
   if (blockIdx.x == 0) {
-    for (int i = threadIdx.x; i < p.K * p.K; i += kPermThreads) p.dispatch[i] = 0;
+    for (int i = threadIdx.x; i < K * K; i += kPermThreads) p.dispatch[i] = 0;
     if (p.expert_counts)
       for (int i = threadIdx.x; i < 2 * p.E; i += kPermThreads) p.expert_counts[i] = 0;
   }
-}
+  __syncthreads();
+  if (threadIdx.x == 0) ok_s = grid_barrier(p.sync, gridDim.x, p.limit_ns, p.status) ? 1 : 0;
+  __syncthreads();
+  if (!ok_s) return;
 
-// One block of 1024 threads; thread b owns block b (n_blocks <= 1024). For every bin, an
-// exclusive scan over blocks gives the block's first position inside the bin; the bin offsets
-// are the exclusive scan of the bin totals.
-__global__ void __launch_bounds__(1024) k_perm_scan(const PermParams p) {
-  __shared__ int wsum[32][kMaxBins];
-  __shared__ int tot[kMaxBins + 1];
-  const int b = threadIdx.x, warp = b >> 5, lane = b & 31;
-  const bool own = b < p.n_blocks;
-  for (int kb = 0; kb < p.K; ++kb) {
-    const int v = own ? p.blk_counts[b * p.K + kb] : 0;
-    int x = v;                                          // inclusive warp scan
+  // offsets: warp w sums bins w, w + 8, ... over all blocks (lanes stride the blocks)
+  for (int kb = warp; kb < K; kb += kPermWarps) {
+    int pre = 0, tot = 0;
+    for (int b = lane; b < p.n_blocks; b += 32) {
+      const int c = __ldcg(p.blk_counts + b * K + kb);
+      tot += c;
+      if (b < static_cast<int>(blockIdx.x)) pre += c;
+    }
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, x, o);
-      if (lane >= o) x += y;
+    for (int o = 16; o > 0; o >>= 1) {
+      pre += __shfl_xor_sync(0xffffffffu, pre, o);
+      tot += __shfl_xor_sync(0xffffffffu, tot, o);
     }
-    if (lane == 31) wsum[warp][kb] = x;
-    if (own) p.blk_offsets[b * p.K + kb] = x - v;       // exclusive within the warp (for now)
+    if (lane == 0) {
+      pre_s[kb] = pre;
+      tot_s[kb] = tot;
+    }
   }
   __syncthreads();
-  if (b < p.K) {                                        // scan warp totals for bin b
+  if (threadIdx.x == 0) {
     int run = 0;
-    for (int w = 0; w < 32; ++w) {
-      const int t = wsum[w][b];
-      wsum[w][b] = run;
-      run += t;
+    for (int kb = 0; kb < K; ++kb) {
+      base[kb] = run + pre_s[kb];
+      if (blockIdx.x == 0) p.bin_offsets[kb] = run;
+      run += tot_s[kb];
     }
-    tot[b] = run;
+    if (blockIdx.x == 0) p.bin_offsets[K] = run;
   }
   __syncthreads();
-  if (b == 0) {
-    int run = 0;
-    for (int kb = 0; kb < p.K; ++kb) {
-      const int t = tot[kb];
-      tot[kb] = run;
-      p.bin_offsets[kb] = run;
-      run += t;
-    }
-    p.bin_offsets[p.K] = run;
-  }
-  __syncthreads();
-  if (own)
-    for (int kb = 0; kb < p.K; ++kb) p.blk_offsets[b * p.K + kb] += wsum[warp][kb] + tot[kb];
-}
 
-__global__ void __launch_bounds__(kPermThreads) k_perm_scatter(const PermParams p) {
-  __shared__ int wcnt[kPermThreads / 32][kMaxBins];
-  __shared__ int base[kMaxBins];
-  __shared__ int disp[kMaxBins * kMaxBins];
-  __shared__ int ecnt[2 * kMaxExperts];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int i = threadIdx.x; i < p.K * p.K; i += kPermThreads) disp[i] = 0;
-  for (int i = threadIdx.x; i < 2 * p.E; i += kPermThreads) ecnt[i] = 0;
-  if (threadIdx.x < p.K) base[threadIdx.x] = p.blk_offsets[blockIdx.x * p.K + threadIdx.x];
-  __syncthreads();
+  // scatter: per round, warp counts per bin -> exclusive scan over warps -> ballot ranks
   const unsigned lt_mask = (1u << lane) - 1u;
   for (int r = 0; r < p.rounds; ++r) {
     const int j = (blockIdx.x * p.rounds + r) * kPermThreads + threadIdx.x;
     const bool valid = j < p.T;
     TokenSel s;
     s.bins = 0u;
-    if (valid) load_sel(p, j, s);
+    if (valid) load_sel(p, s_bin, j, s);
     int home = 0;
     if (valid) {
-      home = p.home ? p.home[j] : static_cast<int>((static_cast<long long>(j) * p.K) / p.T);
-      if (home < 0 || home >= p.K) {
+      home = p.home ? p.home[j] : static_cast<int>((static_cast<long long>(j) * K) / p.T);
+      if (home < 0 || home >= K) {
         atomicOr(p.status, kStatusData);
         home = -1;
       }
     }
-    // ballots: per bin, rank inside the warp and the warp's count
-    for (int kb = 0; kb < p.K; ++kb) {
+    for (int kb = 0; kb < K; ++kb) {
       const unsigned bal = __ballot_sync(0xffffffffu, (s.bins >> kb) & 1u);
       if (lane == 0) wcnt[warp][kb] = __popc(bal);
     }
     __syncthreads();
-    if (threadIdx.x < p.K) {                            // exclusive scan over warps, per bin
+    if (threadIdx.x < K) {                              // exclusive scan over warps, per bin
       int run = base[threadIdx.x];
-      for (int w = 0; w < kPermThreads / 32; ++w) {
+      for (int w = 0; w < kPermWarps; ++w) {
         const int t = wcnt[w][threadIdx.x];
         wcnt[w][threadIdx.x] = run;
         run += t;
@@ -156,17 +183,17 @@ __global__ void __launch_bounds__(kPermThreads) k_perm_scatter(const PermParams 
       base[threadIdx.x] = run;                          // carried into the next round
     }
     __syncthreads();
-    for (int kb = 0; kb < p.K; ++kb) {
+    for (int kb = 0; kb < K; ++kb) {
       const unsigned bal = __ballot_sync(0xffffffffu, (s.bins >> kb) & 1u);
       if ((s.bins >> kb) & 1u) {
         const int pos = wcnt[warp][kb] + __popc(bal & lt_mask);
         uint32_t mask = 0u;
 #pragma unroll
         for (int i = 0; i < kMaxTopK; ++i)
-          if (i < p.k && s.b[i] == kb) mask |= 1u << p.expert_slot[s.e[i]];
+          if (i < p.k && s.b[i] == kb) mask |= 1u << s_slot[s.e[i]];
         p.perm_token[pos] = j;
         p.perm_mask[pos] = mask;
-        if (home >= 0) atomicAdd(&disp[home * p.K + kb], 1);
+        if (home >= 0) atomicAdd(&disp[home * K + kb], 1);
       }
     }
     if (valid && p.expert_counts) {
@@ -177,13 +204,12 @@ __global__ void __launch_bounds__(kPermThreads) k_perm_scatter(const PermParams 
     }
     __syncthreads();                                    // wcnt reused by the next round
   }
-  for (int i = threadIdx.x; i < p.K * p.K; i += kPermThreads)
+  for (int i = threadIdx.x; i < K * K; i += kPermThreads)
     if (disp[i]) atomicAdd(p.dispatch + i, disp[i]);
   if (p.expert_counts)
     for (int i = threadIdx.x; i < 2 * p.E; i += kPermThreads)
       if (ecnt[i]) atomicAdd(p.expert_counts + i, ecnt[i]);
 }
-
 }  // namespace
 
 // Scratch of the no-allocation permutation entry point (see smoes_bin_permute_noalloc): one copy
@@ -211,11 +237,27 @@ cudaError_t static_perm_scratch(StaticPermScratch** out) {
   return cudaSuccess;
 }
 
-// Rounds of 256 tokens per block: 1 while that keeps the block count <= 1024 (the scan runs in
-// one block of 1024 threads), more for larger batches.
+// Blocks of the permutation: all must be resident at once (the grid barrier), and at most
+// kStaticPermBlocks. Rounds of 256 tokens per block grow once the batch needs more blocks.
+int perm_max_blocks() {
+  static std::mutex mu;
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cached[dev] == 0) {
+    int sms = 0, per_sm = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_perm, kPermThreads, 0) != cudaSuccess)
+      return 1;
+    cached[dev] = std::max(1, std::min(kStaticPermBlocks, sms * per_sm));
+  }
+  return cached[dev];
+}
 int perm_rounds(int T) {
   const int units = (T + kPermThreads - 1) / kPermThreads;
-  return units <= 1024 ? 1 : (units + 1023) / 1024;
+  const int cap = perm_max_blocks();
+  return units <= cap ? 1 : (units + cap - 1) / cap;
 }
 int perm_blocks(int T) {
   const int per = kPermThreads * perm_rounds(T);
@@ -223,11 +265,17 @@ int perm_blocks(int T) {
 }
 
 cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s) {
-  if (p.n_blocks > 1024) return cudaErrorInvalidValue;
-  k_perm_count<<<p.n_blocks, kPermThreads, 0, s>>>(p);
-  k_perm_scan<<<1, 1024, 0, s>>>(p);
-  k_perm_scatter<<<p.n_blocks, kPermThreads, 0, s>>>(p);
-  return cudaGetLastError();
+  if (p.n_blocks > perm_max_blocks()) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(p.n_blocks);
+  cfg.blockDim = dim3(kPermThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;    // every block resident: the barrier is safe
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_perm, p);
 }
 
 }  // namespace smoes

@@ -19,6 +19,16 @@ __device__ __forceinline__ uint64_t global_ns() {
   return t;
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// pdl_trigger: the dependent grid launched next may start now. pdl_wait: blocks until the grid
+// this one depends on has completed and its writes are visible (a no-op without a dependency).
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 // ---------------------------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");

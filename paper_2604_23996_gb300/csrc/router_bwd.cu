@@ -111,13 +111,14 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
     const float2 m = __ldg(reinterpret_cast<const float2*>(p.M) + j);
     dv = m.x - 0.5f;
     dt = m.y - 0.5f;
-    const float* tb = p.ws.tabs + static_cast<size_t>(p.ws.token_sample[j]) * 3 * K;
+    // the sample's coefficient table was written by the forward kernel and is read-only here
+    const float* tb = p.ws.tabs + static_cast<size_t>(__ldg(p.ws.token_sample + j)) * 3 * K;
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
       u[q] = 0.f;
       if (e0 + q < E) {
         const int b = __ldg(p.ws.expert_bin + e0 + q);
-        u[q] = __ldcg(tb + 2 * K + b) + dv * __ldcg(tb + b) + dt * __ldcg(tb + K + b);
+        u[q] = __ldg(tb + 2 * K + b) + dv * __ldg(tb + b) + dt * __ldg(tb + K + b);
       }
     }
   } else {
@@ -505,31 +506,63 @@ k_router_bwd_f32(const BwdParams p) {
   }
 }
 
-// dW[e][c] = (accumulate ? dW[e][c] : 0) + S, S = sum_{g=0}^{G-1} part[g][e][c] in that order
-// (the group sum is formed first, so an existing dW adds one rounding, not G).
-__global__ void k_dw_reduce(const BwdParams p) {
+// dW[e][c] = (accumulate ? dW[e][c] : 0) + S, S = sum_{g=0}^{G-1} part[g][e][c]; the group sum is
+// formed first, so an existing dW adds one rounding, not G. A block covers 32 float4 columns of
+// dW with 8 threads each: thread slice t sums groups [t G/8, (t+1) G/8) in order with all its
+// loads in flight at once, then the 8 slice sums are added in slice order (a fixed tree).
+constexpr int kDwSlices = 8;
+constexpr int kDwCols = 32;
+
+__global__ void __launch_bounds__(kDwSlices * kDwCols) k_dw_reduce(const BwdParams p) {
+  __shared__ float4 part_s[kDwSlices][kDwCols];
   const size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
-  const size_t n4 = n / 4;
-  const size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if ((n & 3) == 0) {
-    if (i >= n4) return;
-    const float4* part = reinterpret_cast<const float4*>(p.ws.dw_part);
-    float4 acc = __ldcg(part + i);
-    for (int g = 1; g < p.groups; ++g) {
-      const float4 v = __ldcg(part + static_cast<size_t>(g) * n4 + i);
-      acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+  const bool vec = (n & 3) == 0;
+  const size_t nv = vec ? n / 4 : n;                       // float4 (or scalar) columns
+  const int col = threadIdx.x % kDwCols, sl = threadIdx.x / kDwCols;
+  const size_t i = static_cast<size_t>(blockIdx.x) * kDwCols + col;
+  const int G = p.groups;
+  const int g0 = sl * G / kDwSlices, g1 = (sl + 1) * G / kDwSlices;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (i < nv) {
+    constexpr int kU = 8;
+    for (int g = g0; g < g1; g += kU) {
+      float4 v[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (g + u < g1) {
+          if (vec) {
+            v[u] = __ldcg(reinterpret_cast<const float4*>(p.ws.dw_part) + static_cast<size_t>(g + u) * nv + i);
+          } else {
+            v[u].x = __ldcg(p.ws.dw_part + static_cast<size_t>(g + u) * nv + i);
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        acc.x += v[u].x; acc.y += v[u].y; acc.z += v[u].z; acc.w += v[u].w;
+      }
     }
-    float4* dW = reinterpret_cast<float4*>(p.dW);
-    if (p.accumulate) {
-      const float4 o = dW[i];
-      acc.x += o.x; acc.y += o.y; acc.z += o.z; acc.w += o.w;
+  }
+  part_s[sl][col] = acc;
+  __syncthreads();
+  if (sl == 0 && i < nv) {
+    float4 t = part_s[0][col];
+#pragma unroll
+    for (int q = 1; q < kDwSlices; ++q) {
+      const float4 u = part_s[q][col];
+      t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
     }
-    dW[i] = acc;
-  } else {
-    if (i >= n) return;
-    float acc = __ldcg(p.ws.dw_part + i);
-    for (int g = 1; g < p.groups; ++g) acc += __ldcg(p.ws.dw_part + static_cast<size_t>(g) * n + i);
-    p.dW[i] = p.accumulate ? p.dW[i] + acc : acc;
+    if (vec) {
+      float4* dW = reinterpret_cast<float4*>(p.dW);
+      if (p.accumulate) {
+        const float4 o = dW[i];
+        t.x += o.x; t.y += o.y; t.z += o.z; t.w += o.w;
+      }
+      dW[i] = t;
+    } else {
+      p.dW[i] = p.accumulate ? p.dW[i] + t.x : t.x;
+    }
   }
 }
 
@@ -570,9 +603,8 @@ cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s) {
 cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s) {
   size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
   if ((n & 3) == 0) n /= 4;
-  const int threads = 256;
-  const int blocks = static_cast<int>((n + threads - 1) / threads);
-  k_dw_reduce<<<blocks, threads, 0, s>>>(p);
+  const int blocks = static_cast<int>((n + kDwCols - 1) / kDwCols);
+  k_dw_reduce<<<blocks, kDwSlices * kDwCols, 0, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -7,8 +7,16 @@
 // that completes the last partial of a sample reduces that sample's joint to P (eq. 13),
 // I (eq. 14) and the backward coefficient table; the one that completes the last sample writes
 // the loss of eq. (15). All reductions run in a fixed order: results are bitwise reproducible.
+//
+// Code that runs once per tile is kept in compact loops: a kernel that streams one or two tiles
+// per SM spends most of its epilogue fetching instructions and waiting on dependent latency,
+// not issuing arithmetic.
 #include <cuda_bf16.h>
 #include <math_constants.h>
+
+#include <cfloat>
+
+#include <type_traits>
 
 #include "device_common.cuh"
 #include "ptx.cuh"
@@ -19,23 +27,63 @@ namespace {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kTileRows = kPieceTokens;      // 128 tokens per tile and per partial-sum piece
-constexpr int kPsStride = kTileRows + 1;     // padded row of the per-bin probability table
+constexpr int kPsStride = kTileRows + 1;     // padded row of the per-bin / per-modality tables
+constexpr int kMaxNV = piece_values(kMaxBins);
 
-// Top-k selection key: the logit's bits mapped to an unsigned order-preserving integer, with
-// the low `ib` bits replaced by (2^ib - 1 - e). Keys order by logit (to 23 - ib mantissa bits,
-// at least 15) and, among equal logits, by ascending expert index.
-__device__ __forceinline__ uint32_t topk_key(float z, int e, uint32_t imask) {
+// Top-k selection key: the logit with its low `ib` mantissa bits replaced by the expert index,
+// (2^ib - 1 - e) for a non-negative logit and e for a negative one, so that as floats the keys
+// order by logit (to 23 - ib mantissa bits, at least 15) and, among equal logits, by ascending
+// expert index. Keys compare with float min/max.
+__device__ __forceinline__ float topk_key(float z, int e, uint32_t imask) {
   const uint32_t u = __float_as_uint(z);
-  const uint32_t o = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-  return (o & ~imask) | (imask - static_cast<uint32_t>(e));
+  const uint32_t low = (u & 0x80000000u) ? static_cast<uint32_t>(e) : imask - static_cast<uint32_t>(e);
+  return __uint_as_float((u & ~imask) | low);
+}
+
+// Expert index and logit (low bits set to the middle of their range, relative error below
+// 2^(ib - 24)) of a key.
+__device__ __forceinline__ int topk_index(float key, uint32_t imask) {
+  const uint32_t u = __float_as_uint(key);
+  return static_cast<int>((u & 0x80000000u) ? (u & imask) : imask - (u & imask));
+}
+__device__ __forceinline__ float topk_logit(float key, uint32_t imask) {
+  return __uint_as_float((__float_as_uint(key) & ~imask) | ((imask + 1u) >> 1));
 }
 
 // Sorted (descending) insertion of key q into tk[0..KM): new[i] = max(tk[i], min(tk[i-1], q)).
 template <int KM>
-__device__ __forceinline__ void topk_push(uint32_t (&tk)[KM], uint32_t q) {
+__device__ __forceinline__ void topk_push(float (&tk)[KM], float q) {
 #pragma unroll
-  for (int i = KM - 1; i > 0; --i) tk[i] = max(tk[i], min(tk[i - 1], q));
-  tk[0] = max(tk[0], q);
+  for (int i = KM - 1; i > 0; --i) tk[i] = fmaxf(tk[i], fminf(tk[i - 1], q));
+  tk[0] = fmaxf(tk[0], q);
+}
+
+// Coefficients of the feature pair (2i, 2i+1) (eqs. 8-9) into shared memory as
+// {ga[2i], ga[2i+1], gb[2i], gb[2i+1]}; returns the pair's terms of -2 gc, NaN for invalid
+// statistics. Not inlined: a CTA evaluates it a few times, so one copy of the code is fetched.
+__device__ __noinline__ float gauss_coef_pair(float2 mv, float2 mt, float2 vv, float2 vt, float4* dst) {
+  float a0, b0, c0, a1, b1, c1;
+  const bool g0 = gauss_coef_feature(mv.x, mt.x, vv.x, vt.x, a0, b0, c0);
+  const bool g1 = gauss_coef_feature(mv.y, mt.y, vv.y, vt.y, a1, b1, c1);
+  *dst = make_float4(a0, a1, b0, b1);
+  return (g0 && g1) ? c0 + c1 : CUDART_NAN_F;
+}
+
+// Transpose-reduce of 32 values per lane: afterwards v[0] of lane l holds the sum over the 32
+// lanes of their v[l] (a fixed butterfly tree, 31 shuffles).
+__device__ __forceinline__ float warp_transpose_sum(float (&v)[32]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int s = 16; s >= 1; s >>= 1) {
+    const bool upper = (lane & s) != 0;
+#pragma unroll
+    for (int i = 0; i < s; ++i) {
+      const float send = upper ? v[i] : v[i + s];
+      const float keep = upper ? v[i + s] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+    }
+  }
+  return v[0];
 }
 
 // Reduces sample s (called by the one warp that completed its last piece): fixed-order sums of
@@ -51,60 +99,55 @@ __device__ __forceinline__ void topk_push(uint32_t (&tk)[KM], uint32_t q) {
 //   P_mk = q_k (1 + eps_mk) / (2 + s_v + s_t),
 //   log(P_mk / (P_m P_k)) = log1p(eps_mk) - log1p((eps_vk + eps_tk)/2) + log1p((s_v + s_t)/2) - log1p(s_m),
 // every term a log1p of a small, directly computed quantity; h_k is formed from second-order
-// differences directly as well (see below).
-constexpr int kReduceRound = 16;             // pieces loaded per round before they are summed
-
-__device__ void sample_reduce(const FwdParams& p, int s) {
+// differences directly as well (see below). `red` is kMaxNV floats of shared scratch; the
+// sample's pieces [pb, pe) and token count n are passed in when already loaded (pb < 0: load).
+__device__ __noinline__ void sample_reduce(const FwdParams& p, int s, float* red, int pb, int pe,
+                                           int nt) {
   const Dims& dm = p.dm;
   const int K = dm.K;
   const int NV = piece_values(K);
   const int lane = threadIdx.x & 31;
-  const int pb = p.ws.sample_pieces[s], pe = p.ws.sample_pieces[s + 1];
-  float acc[6];
-#pragma unroll
-  for (int t = 0; t < 6; ++t) acc[t] = 0.f;
-  const int nval = (NV + 31) / 32;            // values per lane (<= 6)
-  for (int q0 = pb; q0 < pe; q0 += kReduceRound) {
-    const int nq = min(kReduceRound, pe - q0);
-    if (nval <= 3) {
-      float v[kReduceRound][3];
-#pragma unroll
-      for (int u = 0; u < kReduceRound; ++u)
-#pragma unroll
-        for (int t = 0; t < 3; ++t) {
-          const int c = lane + 32 * t;
-          v[u][t] = (u < nq && c < NV) ? __ldcg(p.ws.pieces + static_cast<size_t>(q0 + u) * dm.pstride + c) : 0.f;
-        }
-#pragma unroll
-      for (int u = 0; u < kReduceRound; ++u)
-#pragma unroll
-        for (int t = 0; t < 3; ++t) acc[t] += v[u][t];
-    } else {
-      for (int u = 0; u < nq; ++u)
-#pragma unroll
-        for (int t = 0; t < 6; ++t) {
-          const int c = lane + 32 * t;
-          if (c < NV) acc[t] += __ldcg(p.ws.pieces + static_cast<size_t>(q0 + u) * dm.pstride + c);
-        }
-    }
+  if (pb < 0) {
+    pb = p.ws.sample_pieces[s];
+    pe = p.ws.sample_pieces[s + 1];
+    nt = p.ws.offsets[s + 1] - p.ws.offsets[s];
   }
-  auto fetch = [&](int v) -> float {
-    float r = 0.f;
+  // value blocks c, c+1 (values 32c .. 32c+63): lane l loads the blocks of piece q0 + l, a
+  // butterfly sums the 32 pieces of each block, rounds of 32 pieces are added in order
+#pragma unroll 1
+  for (int c = 0; c * 32 < NV; c += 2) {
+    float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll 1
+    for (int q0 = pb; q0 < pe; q0 += 32) {
+      float v0[32], v1[32];
+      const int q = q0 + lane;
+      const float* src = p.ws.pieces + static_cast<size_t>(q) * dm.pstride + 32 * c;
 #pragma unroll
-    for (int t = 0; t < 6; ++t) {
-      const float x = __shfl_sync(0xffffffffu, acc[t], v & 31);
-      if ((v >> 5) == t) r = x;
+      for (int i = 0; i < 16; ++i) {
+        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (q < pe && 32 * c + 4 * i < dm.pstride) f = __ldcg(reinterpret_cast<const float4*>(src + 4 * i));
+        float* v = i < 8 ? v0 + 4 * i : v1 + 4 * (i - 8);
+        v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
+      }
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {           // row padding past the values
+        if (32 * c + i >= NV) v0[i] = 0.f;
+        if (32 * c + 32 + i >= NV) v1[i] = 0.f;
+      }
+      acc0 += warp_transpose_sum(v0);
+      if (32 * c + 32 < NV) acc1 += warp_transpose_sum(v1);
     }
-    return r;
-  };
+    if (32 * c + lane < NV) red[32 * c + lane] = acc0;
+    if (32 * c + 32 + lane < NV) red[32 * c + 32 + lane] = acc1;
+  }
+  __syncwarp();
   const bool act = lane < K;
   const int kk = act ? lane : 0;
-  const float Qall = fetch(kk);                // every lane takes part in the shuffles
-  const float Q = act ? Qall : 0.f;
-  const float Rv = fetch(K + kk), Rt = fetch(2 * K + kk);
-  const float Nv = fetch(3 * K + kk), Nt = fetch(4 * K + kk);
-  const float Dv = fetch(5 * K), Dt = fetch(5 * K + 1), Avd = fetch(5 * K + 2), Atd = fetch(5 * K + 3);
-  const float n = static_cast<float>(p.ws.offsets[s + 1] - p.ws.offsets[s]);
+  const float Q = act ? red[kk] : 0.f;
+  const float Rv = red[K + kk], Rt = red[2 * K + kk];
+  const float Nv = red[3 * K + kk], Nt = red[4 * K + kk];
+  const float Dv = red[5 * K], Dt = red[5 * K + 1], Avd = red[5 * K + 2], Atd = red[5 * K + 3];
+  const float n = static_cast<float>(nt);
   const float sumQ = warp_sum(Q);
   const float q = act ? Q / sumQ : 0.f;
   // per-modality mass and deviation of rho from 1
@@ -112,19 +155,17 @@ __device__ void sample_reduce(const FwdParams& p, int s) {
   const float Av = cv ? 0.5f * n + Dv : Avd;
   const float At = ct ? 0.5f * n + Dt : Atd;
   const bool has_v = Av > 1e-12f, has_t = At > 1e-12f;   // absent modality: Sbar row = 0
+  const float yv = 2.f * Dv / n, yt = 2.f * Dt / n;
   float ev = 0.f, et = 0.f;
-  if (act && has_v) {
-    if (cv) { const float y = 2.f * Dv / n; ev = (2.f * Rv / Q - y) / (1.f + y); }
-    else    { ev = Nv * n / (Q * Av) - 1.f; }
-  }
-  if (act && has_t) {
-    if (ct) { const float y = 2.f * Dt / n; et = (2.f * Rt / Q - y) / (1.f + y); }
-    else    { et = Nt * n / (Q * At) - 1.f; }
-  }
+  if (act && has_v) ev = cv ? (2.f * Rv / Q - yv) / (1.f + yv) : Nv * n / (Q * Av) - 1.f;
+  if (act && has_t) et = ct ? (2.f * Rt / Q - yt) / (1.f + yt) : Nt * n / (Q * At) - 1.f;
   const float sv = warp_sum(q * ev), st = warp_sum(q * et);
   const float NB = static_cast<float>(dm.N_B);
   float Pv = 0.f, Pt = 0.f, a = 0.f, b = 0.f, h = 0.f, I = 0.f;
-  if (has_v && has_t) {
+  if (K == 1) {                      // one bin carries no information: I = 0, P = 1/2 or 1
+    Pv = has_v ? (has_t ? 0.5f : 1.f) : 0.f;
+    Pt = has_t ? (has_v ? 0.5f : 1.f) : 0.f;
+  } else if (has_v && has_t) {
     const float nbz = 2.f + sv + st;                               // N_B * Z
     Pv = q * (1.f + ev) / nbz;                                     // eq. (13)
     Pt = q * (1.f + et) / nbz;
@@ -133,13 +174,12 @@ __device__ void sample_reduce(const FwdParams& p, int s) {
     const float Lt = act ? log1pf(et) - lk + lz - log1pf(st) : 0.f;
     I = warp_sum(Pv * Lv + Pt * Lt);                               // eq. (14)
     const float Z = nbz / NB;
-    a = act ? (Lv - I) / Z / (NB * Av) : 0.f;
-    b = act ? (Lt - I) / Z / (NB * At) : 0.f;
+    a = act ? (Lv - I) / (Z * NB * Av) : 0.f;
+    b = act ? (Lt - I) / (Z * NB * At) : 0.f;
     if (cv && ct && act) {
       // h = (a + b) / 2 is second order (a ~ -b): form L_v + L_t and 1/A_v - 1/A_t directly,
       //   L_v + L_t = log1p(-(d/(1+m))^2) - log1p(-(d_s/(1+m_s))^2),
       // with m, d the half-sum and half-difference of (eps_v, eps_t) and m_s, d_s those of (s_v, s_t).
-      const float yv = 2.f * Dv / n, yt = 2.f * Dt / n;
       const float m = 0.5f * (ev + et), dd = 0.5f * (ev - et);
       const float ms = 0.5f * (sv + st), ds = 0.5f * (sv - st);
       const float rk = dd / (1.f + m), rs = ds / (1.f + ms);
@@ -189,99 +229,183 @@ __device__ void sample_reduce(const FwdParams& p, int s) {
   }
 }
 
-// Shared memory used by the per-tile epilogue group (128 threads, one token row each).
-struct EpiSmem {
-  float* p_s;            // [2][K][kPsStride] bin probabilities of the tile's rows
-  float* m_s;            // [2][4][128] (M_v - 1/2, M_t - 1/2, M_v, M_t) of the tile's rows
-  uint64_t* bar_in;      // count 128: the tile's rows are in p_s / m_s
-  uint64_t* bar_out;     // count 128: the tile's pieces are written
-  const int* s_bin;      // [E]
+// Metadata of one tile, loaded while its accumulator is still being computed: each item is a
+// dependent global load that would otherwise sit on the tile's critical path.
+struct TileMeta {
+  int s0, s1;            // samples of the tile's first and last rows
+  int pbase;             // first partial-sum piece of the tile
+  int row_sample;        // sample of this thread's row, -1 past T
+  int pb0, pe0, n0;      // pieces [pb, pe) and token count of sample s0
+  int pb1, pe1, n1;      // the same for sample s1
 };
 
-// Per-tile epilogue. Provider::load32(c, v) returns logits [32c, 32c+32) of this thread's row
-// (warp-collective; Provider::ncols = logits available, a multiple of 16); release() is called
-// after the last logit read. row: token row in the tile; etid: 0..127 inside the group;
-// lt: index of the tile among those this group processes (selects buffers and phases).
-template <int KM, class Provider, class Release>
-__device__ void epilogue_tile(const FwdParams& p, const Provider& prov, const Release& release,
-                              int tile, int row, int etid, int lt, float dll, const EpiSmem& es,
-                              const WaitCtx& wc) {
+__device__ __forceinline__ TileMeta load_tile_meta(const FwdParams& p, int tile, int row) {
+  const Dims& dm = p.dm;
+  const int t0 = tile * kTileRows;
+  TileMeta m;
+  m.row_sample = t0 + row < dm.T ? __ldg(p.ws.token_sample + t0 + row) : -1;
+  m.s0 = __ldg(p.ws.token_sample + t0);
+  m.s1 = __ldg(p.ws.token_sample + min(t0 + kTileRows - 1, dm.T - 1));
+  m.pbase = __ldg(p.ws.piece_base + tile);
+  m.pb0 = __ldg(p.ws.sample_pieces + m.s0);
+  m.pe0 = __ldg(p.ws.sample_pieces + m.s0 + 1);
+  m.n0 = __ldg(p.ws.offsets + m.s0 + 1) - __ldg(p.ws.offsets + m.s0);
+  m.pb1 = __ldg(p.ws.sample_pieces + m.s1);
+  m.pe1 = __ldg(p.ws.sample_pieces + m.s1 + 1);
+  m.n1 = __ldg(p.ws.offsets + m.s1 + 1) - __ldg(p.ws.offsets + m.s1);
+  return m;
+}
+
+// Shared memory of the per-tile epilogue group (128 threads, one token row each; each warp
+// reads and writes only its own 32 rows of p_s and m_s).
+struct EpiSmem {
+  float* p_s;            // [K][kPsStride] bin probabilities of the tile's rows
+  float* m_s;            // [5][kPsStride] (M_v - 1/2, M_t - 1/2, M_v, M_t, 1) of the tile's rows
+  float* wpart;          // [2][4][kMaxNV] per-warp partial piece sums (double buffer)
+  float* red;            // [kMaxNV] sample-reduce scratch of the group's first warp
+  uint64_t* bar_in;      // count 128: the warps' partials of one (tile, sample) are written
+  uint64_t* bar_out;     // count 128: the tile's pieces are written
+  // optional staging of the tile's softmax scores for one coalesced TMA store: 32-column blocks
+  // of [128 rows][128 bytes], 16-byte chunks swizzled by row (the 128-byte TMA swizzle)
+  uint8_t* stg;          // null: scores are stored row by row
+  uint64_t* stg_full;    // count 128: all rows staged
+  uint64_t* stg_free;    // count 1: the previous tile's store has read the staging
+  const CUtensorMap* tmG;
+};
+
+__host__ __device__ inline size_t epi_smem_floats(int K) {
+  return static_cast<size_t>(K) * kPsStride + 5u * kPsStride + 2u * 4u * kMaxNV + kMaxNV;
+}
+
+__device__ inline EpiSmem epi_smem(float* base, int K, uint64_t* bar_in, uint64_t* bar_out) {
+  EpiSmem es;
+  es.p_s = base;
+  es.m_s = es.p_s + K * kPsStride;
+  es.wpart = es.m_s + 5 * kPsStride;
+  es.red = es.wpart + 2 * 4 * kMaxNV;
+  es.bar_in = bar_in;
+  es.bar_out = bar_out;
+  es.stg = nullptr;
+  es.stg_full = es.stg_free = nullptr;
+  es.tmG = nullptr;
+  return es;
+}
+
+// Per-tile epilogue. Src::load16(c, v) returns logits [16c, 16c+16) of this thread's row,
+// -FLT_MAX past E (finite, so that its top-k key is not a NaN; warp-collective); release() is
+// called after the last logit read. row: token row in
+// the tile (0..127, the thread's index in the group); lt: index of the tile among those this
+// group processes; meta: the tile's metadata (load_tile_meta); n_in: completed phases of
+// bar_in (identical in all 128 threads).
+template <int KM, class Src, class Release>
+__device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release& release, int tile,
+                              int row, int lt, float dll, const TileMeta& meta, const EpiSmem& es,
+                              const WaitCtx& wc, uint32_t& n_in) {
   const Dims& dm = p.dm;
   const int E = dm.E, K = dm.K, k = dm.k;
+  const int wg = row >> 5, lane = row & 31;
   const int j = tile * kTileRows + row;
   const bool valid = j < dm.T;
-  const int buf = lt & 1;
-  float* p_s = es.p_s + buf * K * kPsStride;
-  float* m_s = es.m_s + buf * 4 * kTileRows;
-  const uint32_t imask = (E <= 2) ? 1u : ((1u << (32 - __clz(E - 1))) - 1u);
-  const int nch = (prov.ncols + 31) / 32;
+  const int nch = (E + 15) >> 4;
+  const uint32_t imask = (1u << (32 - __clz(max(nch * 16 - 1, 1)))) - 1u;
 
-  // pass 1: softmax max and top-k keys
-  uint32_t tk[KM];
+  // pass A: softmax max and top-k keys, even and odd columns in two independent lists (two
+  // dependency chains), merged at the end
+  float tk[KM], tk2[KM];
 #pragma unroll
-  for (int i = 0; i < KM; ++i) tk[i] = 0u;
-  float mx = -CUDART_INF_F;
+  for (int i = 0; i < KM; ++i) tk[i] = tk2[i] = -CUDART_INF_F;
+  float mx = -CUDART_INF_F, mx2 = -CUDART_INF_F;
+#pragma unroll 1
   for (int c = 0; c < nch; ++c) {
-    float v[32];
-    prov.load32(c, v);
+    float v[16];
+    src.load16(c, v);
 #pragma unroll
-    for (int t = 0; t < 32; ++t) {
-      const int e = c * 32 + t;
-      if (e < E) {
-        mx = fmaxf(mx, v[t]);
-        topk_push<KM>(tk, topk_key(v[t], e, imask));
-      }
+    for (int t = 0; t < 16; t += 2) {
+      mx = fmaxf(mx, v[t]);
+      mx2 = fmaxf(mx2, v[t + 1]);
+      topk_push<KM>(tk, topk_key(v[t], c * 16 + t, imask));
+      topk_push<KM>(tk2, topk_key(v[t + 1], c * 16 + t + 1, imask));
     }
   }
-  // pass 2: softmax denominator
-  float sum = 0.f;
-  for (int c = 0; c < nch; ++c) {
-    float v[32];
-    prov.load32(c, v);
+  mx = fmaxf(mx, mx2);
 #pragma unroll
-    for (int t = 0; t < 32; ++t)
-      if (c * 32 + t < E) sum += exp2f((v[t] - mx) * kLog2e);
+  for (int i = 0; i < KM; ++i) topk_push<KM>(tk, tk2[i]);
+  // pass B: softmax denominator (four partial sums, added in a fixed order)
+  const float mxl = mx * kLog2e;
+  float sum = 0.f;
+#pragma unroll 1
+  for (int c = 0; c < nch; ++c) {
+    float v[16];
+    src.load16(c, v);
+    float ps[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int t = 0; t < 16; ++t) ps[t & 3] += exp2f(fmaf(v[t], kLog2e, -mxl));
+    sum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
   }
   const float inv = 1.f / sum;
   if (valid && !(isfinite(mx) && isfinite(sum) && sum > 0.f)) atomicOr(p.ws.status, kStatusData);
-  // pass 3: g, saved g, bin sums (accumulated over runs of experts sharing a bin)
-  for (int kb = 0; kb < K; ++kb) p_s[kb * kPsStride + row] = 0.f;
+  // pass C: g, saved g, bin probabilities
   float* grow = p.ws.gsave + static_cast<size_t>(valid ? j : 0) * E;
+  float* prow = es.p_s + row;                       // p_s[b][row] at prow[b * kPsStride]
   const bool vec = (E & 3) == 0;
+  const bool stg = es.stg != nullptr;
   float run = 0.f;
-  int run_bin = es.s_bin[0];
+  int cnt = 0, bin = 0;
+  if (!dm.contig_bins)
+    for (int b = 0; b < K; ++b) prow[b * kPsStride] = 0.f;
+  if (stg && lt > 0 && !mbar_wait(es.stg_free, static_cast<uint32_t>((lt - 1) & 1), wc)) return;
+#pragma unroll 1
   for (int c = 0; c < nch; ++c) {
-    float v[32];
-    prov.load32(c, v);
+    float v[16];
+    src.load16(c, v);
 #pragma unroll
-    for (int t = 0; t < 32; ++t) v[t] = (c * 32 + t < E) ? exp2f((v[t] - mx) * kLog2e) * inv : 0.f;
-    if (valid) {
-      if (vec && c * 32 + 32 <= E) {
+    for (int t = 0; t < 16; ++t) v[t] = exp2f(fmaf(v[t], kLog2e, -mxl)) * inv;
+    if (stg) {
+      uint8_t* rb = es.stg + (c >> 1) * 16384 + row * 128;
 #pragma unroll
-        for (int t = 0; t < 32; t += 4)
-          *reinterpret_cast<float4*>(grow + c * 32 + t) = make_float4(v[t], v[t + 1], v[t + 2], v[t + 3]);
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t qd = static_cast<uint32_t>((c & 1) * 4 + i);
+        *reinterpret_cast<float4*>(rb + ((qd ^ static_cast<uint32_t>(row & 7)) << 4)) =
+            make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+      }
+    } else if (valid) {
+      if (vec && c * 16 + 16 <= E) {
+#pragma unroll
+        for (int t = 0; t < 16; t += 4)
+          *reinterpret_cast<float4*>(grow + c * 16 + t) = make_float4(v[t], v[t + 1], v[t + 2], v[t + 3]);
       } else {
 #pragma unroll
-        for (int t = 0; t < 32; ++t)
-          if (c * 32 + t < E) grow[c * 32 + t] = v[t];
+        for (int t = 0; t < 16; ++t)
+          if (c * 16 + t < E) grow[c * 16 + t] = v[t];
       }
     }
+    if (dm.contig_bins) {              // bins are runs of N_B experts, N_B a multiple of 4
 #pragma unroll
-    for (int t = 0; t < 32; ++t) {
-      const int e = c * 32 + t;
-      if (e < E) {
-        const int b = es.s_bin[e];                 // warp-uniform
-        if (b != run_bin) {
-          p_s[run_bin * kPsStride + row] += run;
+      for (int q = 0; q < 4; ++q) {
+        run += (v[4 * q] + v[4 * q + 1]) + (v[4 * q + 2] + v[4 * q + 3]);
+        cnt += 4;
+        if (cnt == dm.N_B) {
+          if (bin < K) prow[bin * kPsStride] = run;
           run = 0.f;
-          run_bin = b;
+          cnt = 0;
+          ++bin;
         }
-        run += v[t];
       }
+    } else {                           // any expert -> bin map
+#pragma unroll
+      for (int t = 0; t < 16; ++t)
+        if (c * 16 + t < E) prow[__ldg(p.ws.expert_bin + c * 16 + t) * kPsStride] += v[t];
     }
   }
-  p_s[run_bin * kPsStride + row] += run;
   release();
+  if (stg) {                       // one thread stores the staged scores (rows >= T are clipped)
+    fence_proxy_async_smem();
+    mbar_arrive(es.stg_full);
+    if (row == 0 && mbar_wait(es.stg_full, static_cast<uint32_t>(lt & 1), wc)) {
+      for (int b = 0; b * 32 < E; ++b) tma_store_2d(es.tmG, es.stg + b * 16384, 32 * b, tile * kTileRows);
+      tma_store_commit();
+    }
+  }
 
   // modality score of this token (eq. 9 for two modalities, or the provided scores)
   float Mv = 0.f, Mt = 0.f, dv = 0.f, dt = 0.f;
@@ -300,161 +424,146 @@ __device__ void epilogue_tile(const FwdParams& p, const Provider& prov, const Re
       dt = -dv;
       if (p.M_out) reinterpret_cast<float2*>(p.M_out)[j] = make_float2(Mv, Mt);
     }
-    // top-k outputs: indices from the keys, weights = the exact saved scores
+    // top-k outputs: indices from the keys; weights = the staged scores, or recomputed from the
+    // keys' logits when the scores are not staged
     float w[KM];
     float wsum = 0.f;
 #pragma unroll
     for (int i = 0; i < KM; ++i) {
       w[i] = 0.f;
       if (i < k) {
-        const int e = static_cast<int>(imask - (tk[i] & imask));
-        p.topk_idx[static_cast<size_t>(j) * k + i] = e;
-        w[i] = grow[e];
-        wsum += w[i];
-      }
-    }
-    const float ws = dm.renorm ? 1.f / wsum : 1.f;
-#pragma unroll
-    for (int i = 0; i < KM; ++i)
-      if (i < k) p.topk_w[static_cast<size_t>(j) * k + i] = w[i] * ws;
-    if (p.bin_prob)
-      for (int kb = 0; kb < K; ++kb) p.bin_prob[static_cast<size_t>(j) * K + kb] = p_s[kb * kPsStride + row];
-  }
-  m_s[0 * kTileRows + row] = dv;
-  m_s[1 * kTileRows + row] = dt;
-  m_s[2 * kTileRows + row] = Mv;
-  m_s[3 * kTileRows + row] = Mt;
-  mbar_arrive(es.bar_in);
-  if (!mbar_wait(es.bar_in, static_cast<uint32_t>(lt & 1), wc)) return;
-
-  // partial sums of the joint table: one piece per (tile, sample), fixed row order
-  const int t0 = tile * kTileRows;
-  const int s0 = p.ws.token_sample[t0];
-  const int s1 = p.ws.token_sample[min(t0 + kTileRows - 1, dm.T - 1)];
-  const int NV = piece_values(K);
-  const int pbase = p.ws.piece_base[tile];
-  for (int s = s0; s <= s1; ++s) {
-    const int r0 = max(p.ws.offsets[s] - t0, 0);
-    const int r1 = min(p.ws.offsets[s + 1] - t0, kTileRows);
-    float* piece = p.ws.pieces + static_cast<size_t>(pbase + (s - s0)) * dm.pstride;
-    for (int v = etid; v < NV; v += 128) {
-      float acc = 0.f;
-      if (v < 5 * K) {
-        const int kind = v / K, kb = v - kind * K;
-        const float* pr = p_s + kb * kPsStride;
-        if (kind == 0) {
-          for (int r = r0; r < r1; ++r) acc += pr[r];
+        if (stg) {
+          const uint32_t e = static_cast<uint32_t>(topk_index(tk[i], imask));
+          const uint32_t qd = ((e & 31u) >> 2) ^ static_cast<uint32_t>(row & 7);
+          w[i] = *reinterpret_cast<const float*>(es.stg + (e >> 5) * 16384u + row * 128 + (qd << 4) + (e & 3u) * 4u);
         } else {
-          const float* wr = m_s + (kind - 1) * kTileRows;
-          for (int r = r0; r < r1; ++r) acc = fmaf(wr[r], pr[r], acc);
+          w[i] = exp2f(fmaf(topk_logit(tk[i], imask), kLog2e, -mxl)) * inv;
         }
-      } else {
-        const float* wr = m_s + (v - 5 * K) * kTileRows;
-        for (int r = r0; r < r1; ++r) acc += wr[r];
       }
-      piece[v] = acc;
+      wsum += w[i];
     }
+    const float wsc = dm.renorm ? 1.f / wsum : 1.f;
+    int32_t* ti = p.topk_idx + static_cast<size_t>(j) * k;
+    float* tw = p.topk_w + static_cast<size_t>(j) * k;
+#pragma unroll
+    for (int i = 0; i < KM; ++i) {
+      if (i < k) {
+        ti[i] = topk_index(tk[i], imask);
+        tw[i] = w[i] * wsc;
+      }
+    }
+    if (p.bin_prob)
+      for (int kb = 0; kb < K; ++kb) p.bin_prob[static_cast<size_t>(j) * K + kb] = prow[kb * kPsStride];
+  } else {
+    for (int b = 0; b < K; ++b) prow[b * kPsStride] = 0.f;
+  }
+  float* mrow = es.m_s + row;
+  mrow[0] = dv;
+  mrow[kPsStride] = dt;
+  mrow[2 * kPsStride] = Mv;
+  mrow[3 * kPsStride] = Mt;
+  mrow[4 * kPsStride] = 1.f;
+  __syncwarp();
+
+  // partial sums of the joint table: one piece per (tile, sample); each warp sums its 32 rows
+  // (lane = value), the four warp partials are then added in warp order. The rows of a sample
+  // are contiguous: a ballot over the rows' sample ids gives the warp's range.
+  const int NV = piece_values(K);
+  const int s0 = meta.s0, s1 = meta.s1;
+  for (int s = s0; s <= s1; ++s) {
+    const uint32_t mine = __ballot_sync(0xffffffffu, meta.row_sample == s);
+    const int r0 = 32 * wg + (mine ? __ffs(mine) - 1 : 0);
+    const int r1 = 32 * wg + (mine ? 32 - __clz(mine) : 0);
+    float* wp = es.wpart + ((n_in & 1) * 4 + wg) * kMaxNV;
+    for (int v = lane; v < NV; v += 32) {
+      // value v: kind v / K over bin v % K (kind 0: Q, 1..4: weighted by m_s rows 0..3),
+      // or, past 5K, the plain sum of m_s row v - 5K
+      const int kind = v < 5 * K ? v / K : 0;
+      const float* a = v < 5 * K ? es.p_s + (v - kind * K) * kPsStride : es.m_s + (v - 5 * K) * kPsStride;
+      const float* w = es.m_s + (v < 5 * K ? (kind + 4) % 5 : 4) * kPsStride;
+      float acc = 0.f;
+#pragma unroll 4
+      for (int r = r0; r < r1; ++r) acc = fmaf(w[r], a[r], acc);
+      wp[v] = acc;
+    }
+    mbar_arrive(es.bar_in);
+    if (!mbar_wait(es.bar_in, n_in & 1u, wc)) return;
+    const float* w0 = es.wpart + (n_in & 1) * 4 * kMaxNV;
+    ++n_in;
+    float* piece = p.ws.pieces + static_cast<size_t>(meta.pbase + (s - s0)) * dm.pstride;
+    for (int v = row; v < NV; v += 128)
+      piece[v] = ((w0[v] + w0[kMaxNV + v]) + w0[2 * kMaxNV + v]) + w0[3 * kMaxNV + v];
+  }
+  if (stg && row == 0) {            // the staging may be rewritten once the store has read it
+    tma_store_wait_read<0>();
+    mbar_arrive(es.stg_free);
   }
   __threadfence();
   mbar_arrive(es.bar_out);
-  if (etid < 32) {                        // one warp announces the pieces and reduces samples
-    const int lane = threadIdx.x & 31;
+  if (wg == 0) {                        // the first warp announces the pieces, reduces samples
     bool ok = true;
     if (lane == 0) ok = mbar_wait(es.bar_out, static_cast<uint32_t>(lt & 1), wc);
     ok = __shfl_sync(0xffffffffu, ok, 0);
     if (!ok) return;
     for (int s = s0; s <= s1; ++s) {
+      // a sample strictly inside the tile has this tile's piece only
+      const int pb = s == s0 ? meta.pb0 : s == s1 ? meta.pb1 : meta.pbase + (s - s0);
+      const int pe = s == s0 ? meta.pe0 : s == s1 ? meta.pe1 : pb + 1;
+      const int nt = s == s0 ? meta.n0 : s == s1 ? meta.n1 : 0;
       uint32_t last = 0;
-      if (lane == 0) {
-        const uint32_t need = static_cast<uint32_t>(p.ws.sample_pieces[s + 1] - p.ws.sample_pieces[s]);
-        last = (atomicAdd(p.ws.sample_ticket + s, 1u) + 1u == need);
-      }
+      if (lane == 0) last = (atomicAdd(p.ws.sample_ticket + s, 1u) + 1u == static_cast<uint32_t>(pe - pb));
       last = __shfl_sync(0xffffffffu, last, 0);
       if (last) {
         __threadfence();
-        sample_reduce(p, s);
+        const bool known = s == s0 || s == s1;
+        sample_reduce(p, s, es.red, known ? pb : -1, pe, nt);
       }
     }
   }
-}
-
-// Gaussian coefficients computed by the 128 threads of the Gaussian group (gtid 0..127), with
-// the group synchronised through `bar` (count 128). Returns gc in every thread.
-__device__ float gauss_coef_group(const FwdParams& p, int dpad, float* ga, float* gb, float* red,
-                                  uint64_t* bar, int gtid, const WaitCtx& wc) {
-  const int d = p.dm.d;
-  constexpr int kU = 8;                      // elements per thread and round, loads first
-  float part = 0.f;
-  bool bad = false;
-  for (int i0 = gtid; i0 < dpad; i0 += 128 * kU) {
-    float vv[kU], vt[kU], mv[kU], mt[kU];
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int i = i0 + 128 * u;
-      const bool in = i < d;
-      vv[u] = in ? __ldg(p.var + i) : 1.f;
-      vt[u] = in ? __ldg(p.var + d + i) : 1.f;
-      mv[u] = in ? __ldg(p.mu + i) : 0.f;
-      mt[u] = in ? __ldg(p.mu + d + i) : 0.f;
-    }
-#pragma unroll
-    for (int u = 0; u < kU; ++u) {
-      const int i = i0 + 128 * u;
-      if (i >= dpad) break;
-      if (!(vv[u] > 0.f) || !(vt[u] > 0.f) || !isfinite(vv[u]) || !isfinite(vt[u]) ||
-          !isfinite(mv[u]) || !isfinite(mt[u]))
-        bad = true;
-      const float pv = vv[u] * vt[u];
-      ga[i] = (vv[u] - vt[u]) / (2.f * pv);
-      gb[i] = (mv[u] * vt[u] - mt[u] * vv[u]) / pv;
-      if (i < d) part += log1pf((vv[u] - vt[u]) / vt[u]) + (mv[u] * mv[u] * vt[u] - mt[u] * mt[u] * vv[u]) / pv;
-    }
-  }
-  if (bad) atomicOr(p.ws.status, kStatusData);
-  part = warp_sum(part);
-  if ((gtid & 31) == 0) red[gtid >> 5] = part;
-  mbar_arrive(bar);
-  mbar_wait(bar, 0, wc);
-  return -0.5f * (((red[0] + red[1]) + red[2]) + red[3]);
 }
 
 // ------------------------------------------------------------------ tcgen05 forward (bf16)
 
 __host__ __device__ inline size_t fwd_stage_bytes(int N) { return 16384u + static_cast<size_t>(N) * 128u; }
 
-__host__ __device__ inline size_t epi_smem_floats(int K) {
-  return 2u * static_cast<size_t>(K) * kPsStride + 2u * 4u * kTileRows;
-}
+// Staged softmax scores: 32-column blocks of [128 rows][32 floats].
+__host__ __device__ inline size_t fwd_stg_bytes(int E) { return static_cast<size_t>(round_up(E, 32)) * 512u; }
 
-__host__ __device__ inline size_t fwd_smem_bytes(int N, int n_stages, int d, int K, int E, bool gauss) {
+__host__ __device__ inline size_t fwd_smem_bytes(int N, int n_stages, int d, int K, int E, bool gauss,
+                                                 bool stg) {
   size_t b = static_cast<size_t>(n_stages) * fwd_stage_bytes(N);
+  if (stg) b += fwd_stg_bytes(E);
   if (gauss) b += 2u * sizeof(float) * static_cast<size_t>(round_up(d, kFwdBK));
   b += sizeof(float) * (epi_smem_floats(K) + 256u + 8u);
-  b += sizeof(int) * static_cast<size_t>(round_up(E, 4));
-  b += sizeof(uint64_t) * (2u * n_stages + 12u);
+  b += sizeof(uint64_t) * (2u * n_stages + 16u);
   b += 16u;
   return b + 1024u;   // alignment slack
 }
 
+// 10 warps: three share a sub-partition's 16K registers, so a thread gets at most 168.
 template <bool kGauss, int KM>
 __global__ void __launch_bounds__(kGauss ? 320 : 192, 1)
 k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
-                const FwdParams p, const int N, const int n_stages) {
+                const __grid_constant__ CUtensorMap tmG, const FwdParams p, const int N,
+                const int n_stages, const int use_stg) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const Dims& dm = p.dm;
   const int dpad = round_up(dm.d, kFwdBK);
   const int n_kb = dpad / kFwdBK;
+  // CTAs walk the K-blocks from different starting points, so that they do not all request the
+  // same W tile from L2 at the same moment
+  const int kb0 = blockIdx.x % n_kb;
+  auto kb_at = [&](int i) { return (kb0 + i) % n_kb; };
   const size_t sbytes = fwd_stage_bytes(N);
 
   uint8_t* q = base;
   uint8_t* stage = q;                             q += n_stages * sbytes;
-  float* ga = reinterpret_cast<float*>(q);        q += kGauss ? sizeof(float) * dpad : 0;
-  float* gb = reinterpret_cast<float*>(q);        q += kGauss ? sizeof(float) * dpad : 0;
+  uint8_t* stg = q;                               q += use_stg ? fwd_stg_bytes(dm.E) : 0;
+  float4* cq = reinterpret_cast<float4*>(q);      q += kGauss ? 2 * sizeof(float) * dpad : 0;
   float* epi = reinterpret_cast<float*>(q);       q += sizeof(float) * epi_smem_floats(dm.K);
   float* dll_s = reinterpret_cast<float*>(q);     q += sizeof(float) * 256;
-  float* red = reinterpret_cast<float*>(q);       q += sizeof(float) * 8;
-  int* s_bin = reinterpret_cast<int*>(q);         q += sizeof(int) * round_up(dm.E, 4);
+  float* gred = reinterpret_cast<float*>(q);      q += sizeof(float) * 8;
   q = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(q) + 7) & ~uintptr_t(7));
   uint64_t* full = reinterpret_cast<uint64_t*>(q);      q += 8 * n_stages;
   uint64_t* empty = reinterpret_cast<uint64_t*>(q);     q += 8 * n_stages;
@@ -466,6 +575,9 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   uint64_t* bar_in = reinterpret_cast<uint64_t*>(q);    q += 8;
   uint64_t* bar_out = reinterpret_cast<uint64_t*>(q);   q += 8;
   uint64_t* coef_bar = reinterpret_cast<uint64_t*>(q);  q += 8;
+  uint64_t* coef_issued = reinterpret_cast<uint64_t*>(q);  q += 8;
+  uint64_t* stg_full = reinterpret_cast<uint64_t*>(q);  q += 8;
+  uint64_t* stg_free = reinterpret_cast<uint64_t*>(q);  q += 8;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q); q += 4;
   int* abort_flag = reinterpret_cast<int*>(q);
 
@@ -487,12 +599,14 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     mbar_init(drain, 1);
     mbar_init(bar_in, 128);
     mbar_init(bar_out, 128);
-    mbar_init(coef_bar, 128);
+    mbar_init(coef_bar, 256);
+    mbar_init(coef_issued, 256);
+    mbar_init(stg_full, 128);
+    mbar_init(stg_free, 1);
     fence_mbar_init();
     tma_prefetch_desc(&tmX);
     tma_prefetch_desc(&tmW);
   }
-  for (int e = threadIdx.x; e < dm.E; e += blockDim.x) s_bin[e] = p.ws.expert_bin[e];
   const uint32_t tmem_cols = (2 * N <= 32) ? 32u : (2 * N <= 64) ? 64u : (2 * N <= 128) ? 128u
                                                  : (2 * N <= 256) ? 256u : 512u;
   if (warp == 1) tmem_alloc(tmem_slot, tmem_cols);
@@ -500,6 +614,43 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+
+  if (kGauss && warp >= 2) {
+    // this CTA's Gaussian coefficients (eqs. 8-9), computed by the epilogue and Gaussian warps
+    // (256 threads) as feature pairs interleaved as float4 {ga[2i], ga[2i+1], gb[2i], gb[2i+1]};
+    // four pairs per thread and round, loads first; the first round is requested before the
+    // producer starts the X stream
+    const int ct = threadIdx.x - 64;
+    const float2* mu2 = reinterpret_cast<const float2*>(p.mu);
+    const float2* var2 = reinterpret_cast<const float2*>(p.var);
+    const int np = dm.d / 2;
+    float part = 0.f;
+    bool announced = false;
+    for (int i0 = ct; i0 < dpad / 2; i0 += 4 * 256) {
+      float2 mv[4], mt[4], vv[4], vt[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + 256 * u;
+        const bool in = i < np;
+        mv[u] = in ? __ldg(mu2 + i) : make_float2(0.f, 0.f);
+        mt[u] = in ? __ldg(mu2 + np + i) : make_float2(0.f, 0.f);
+        vv[u] = in ? __ldg(var2 + i) : make_float2(1.f, 1.f);
+        vt[u] = in ? __ldg(var2 + np + i) : make_float2(1.f, 1.f);
+      }
+      if (!announced) {
+        mbar_arrive(coef_issued);
+        announced = true;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (i0 + 256 * u < dpad / 2) part += gauss_coef_pair(mv[u], mt[u], vv[u], vt[u], cq + i0 + 256 * u);
+    }
+    if (!announced) mbar_arrive(coef_issued);
+    if (!isfinite(part)) atomicOr(p.ws.status, kStatusData);
+    part = warp_sum(part);
+    if (lane == 0) gred[warp - 2] = part;
+    mbar_arrive(coef_bar);
+  }
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
@@ -509,13 +660,16 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       long issued = 0;
       bool ok = true;
       const uint32_t tx = static_cast<uint32_t>(sbytes);
+      // the Gaussian statistics are requested before the X stream floods the memory system
+      if (kGauss) ok = mbar_wait(coef_issued, 0, wc);
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
         for (int kb = 0; kb < n_kb; ++kb) {
           if (!mbar_wait(empty + st, ph ^ 1u, wc)) { ok = false; break; }
           uint8_t* xs = stage + st * sbytes;
           mbar_arrive_expect_tx(full + st, tx);
-          tma_load_2d(xs, &tmX, full + st, kb * kFwdBK, tile * kFwdBM);
-          tma_load_2d(xs + 16384, &tmW, full + st, kb * kFwdBK, 0);
+          const int kx = kb_at(kb);
+          tma_load_2d(xs, &tmX, full + st, kx * kFwdBK, tile * kFwdBM);
+          tma_load_2d(xs + 16384, &tmW, full + st, kx * kFwdBK, 0);
           ++issued;
           if (++st == n_stages) { st = 0; ph ^= 1u; }
         }
@@ -566,12 +720,36 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     // ---------------------------------------------------------------- epilogue (4 warps)
     const int lg = warp & 3;                 // TMEM lane group accessible to this warp
     const int row = lg * 32 + lane;          // tile row == TMEM lane == token offset
-    const int etid = threadIdx.x - 64;
-    EpiSmem es{epi, epi + 2 * dm.K * kPsStride, bar_in, bar_out, s_bin};
+    EpiSmem es = epi_smem(epi, dm.K, bar_in, bar_out);
+    if (use_stg) {
+      es.stg = stg;
+      es.stg_full = stg_full;
+      es.stg_free = stg_free;
+      es.tmG = &tmG;
+    }
+    struct Src {                    // logits of this warp's rows from TMEM
+      uint32_t base;
+      int E;
+      __device__ void load16(int c, float (&v)[16]) const {
+        tmem_ld16(base + 16u * c, v);
+        if (16 * c + 16 > E) {
+#pragma unroll
+          for (int t = 0; t < 16; ++t)
+            if (16 * c + t >= E) v[t] = -FLT_MAX;
+        }
+      }
+    };
+    struct Rel {                    // hand the accumulator buffer back to the MMA warp
+      uint64_t* bar;
+      __device__ void operator()() const { tc_fence_before(); mbar_arrive(bar); }
+    };
+    const uint32_t tl = tmem_base + (static_cast<uint32_t>(lg * 32) << 16);
+    uint32_t n_in = 0;
     int lt = 0;
     for (int tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x, ++lt) {
       const int buf = lt & 1;
       const uint32_t use = static_cast<uint32_t>(lt >> 1);
+      const TileMeta meta = load_tile_meta(p, tile, row);    // lands while the tile streams in
       if (!mbar_wait(acc_full + buf, use & 1u, wc)) break;
       tc_fence_after();
       float dll = 0.f;
@@ -580,71 +758,53 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
         dll = dll_s[buf * 128 + row];
         mbar_arrive(g_empty + buf);
       }
-      struct Prov {
-        uint32_t base;
-        int ncols;
-        __device__ void load32(int c, float (&v)[32]) const {
-          if (32 * c + 32 <= ncols) {
-            tmem_ld32(base + 32u * c, v);
-          } else {
-            float h[16];
-            tmem_ld16(base + 32u * c, h);
-#pragma unroll
-            for (int i = 0; i < 16; ++i) { v[i] = h[i]; v[16 + i] = 0.f; }
-          }
-        }
-      } prov{tmem_base + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(buf * N), N};
-      struct Rel {                  // hand the accumulator buffer back to the MMA warp
-        uint64_t* bar;
-        __device__ void operator()() const { tc_fence_before(); mbar_arrive(bar); }
-      } rel{acc_empty + buf};
-      epilogue_tile<KM>(p, prov, rel, tile, row, etid, lt, dll, es, wc);
+      epilogue_tile<KM>(p, Src{tl + static_cast<uint32_t>(buf * N), dm.E}, Rel{acc_empty + buf},
+                        tile, row, lt, dll, meta, es, wc, n_in);
     }
+    if (use_stg && row == 0) tma_store_wait_all<0>();   // the score stores complete before exit
   } else {
     // ---------------------------------------------------------------- Gaussian warps (4)
+    // Warp w owns tile rows 32w..32w+31 and lane l the feature pair (2l, 2l+1) of every K-block:
+    // per stage a lane reads one float4 of coefficients and one 4-byte word of each of its
+    // warp's rows, and keeps one running sum per row; a butterfly over the lanes gives the row
+    // totals at the end of the tile.
     if (kGauss) {
-      const int row = (warp - 6) * 32 + lane;
-      const float gc = gauss_coef_group(p, dpad, ga, gb, red, coef_bar, row, wc);
+      const int gw = warp - 6;
+      const int gt = gw * 32 + lane;
+      bool ok = mbar_wait(coef_bar, 0, wc);
+      float gc = 0.f;
+      for (int w = 0; w < 8; ++w) gc += gred[w];
+      gc *= -0.5f;
+      // byte offset of this lane's word inside a 128-byte swizzled row r: chunk (l/4) ^ (r & 7)
+      const uint32_t wcol = static_cast<uint32_t>(lane & 3) * 4u;
+      const uint32_t chk = static_cast<uint32_t>(lane >> 2);
       int st = 0;
       uint32_t ph = 0;
       int lt = 0;
-      bool ok = true;
       for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++lt) {
         const int buf = lt & 1;
         const uint32_t use = static_cast<uint32_t>(lt >> 1);
         if (!mbar_wait(g_empty + buf, (use & 1u) ^ 1u, wc)) break;
-        float acc = 0.f;
+        float acc[32];
+#pragma unroll
+        for (int r = 0; r < 32; ++r) acc[r] = 0.f;
         for (int kb = 0; kb < n_kb; ++kb) {
           if (!mbar_wait(full + st, ph, wc)) { ok = false; break; }
-          const uint8_t* xr = stage + st * sbytes + row * 128;
-          const float* a = ga + kb * kFwdBK;
-          const float* b = gb + kb * kFwdBK;
+          const uint8_t* xs = stage + st * sbytes + gw * 32 * 128;
+          const float4 cf = cq[kb_at(kb) * 32 + lane];
 #pragma unroll
-          for (int c = 0; c < 8; ++c) {
-            const uint4 u = *reinterpret_cast<const uint4*>(xr + ((c ^ (row & 7)) << 4));
-            const float4 a0 = *reinterpret_cast<const float4*>(a + c * 8);
-            const float4 a1 = *reinterpret_cast<const float4*>(a + c * 8 + 4);
-            const float4 b0 = *reinterpret_cast<const float4*>(b + c * 8);
-            const float4 b1 = *reinterpret_cast<const float4*>(b + c * 8 + 4);
-            const float x0 = __uint_as_float(u.x << 16), x1 = __uint_as_float(u.x & 0xffff0000u);
-            const float x2 = __uint_as_float(u.y << 16), x3 = __uint_as_float(u.y & 0xffff0000u);
-            const float x4 = __uint_as_float(u.z << 16), x5 = __uint_as_float(u.z & 0xffff0000u);
-            const float x6 = __uint_as_float(u.w << 16), x7 = __uint_as_float(u.w & 0xffff0000u);
-            acc = fmaf(x0, fmaf(a0.x, x0, b0.x), acc);
-            acc = fmaf(x1, fmaf(a0.y, x1, b0.y), acc);
-            acc = fmaf(x2, fmaf(a0.z, x2, b0.z), acc);
-            acc = fmaf(x3, fmaf(a0.w, x3, b0.w), acc);
-            acc = fmaf(x4, fmaf(a1.x, x4, b1.x), acc);
-            acc = fmaf(x5, fmaf(a1.y, x5, b1.y), acc);
-            acc = fmaf(x6, fmaf(a1.z, x6, b1.z), acc);
-            acc = fmaf(x7, fmaf(a1.w, x7, b1.w), acc);
+          for (int r = 0; r < 32; ++r) {
+            const uint32_t u = *reinterpret_cast<const uint32_t*>(xs + r * 128 + ((chk ^ (r & 7)) << 4) + wcol);
+            const float x0 = __uint_as_float(u << 16), x1 = __uint_as_float(u & 0xffff0000u);
+            acc[r] = fmaf(x0, fmaf(cf.x, x0, cf.z), acc[r]);
+            acc[r] = fmaf(x1, fmaf(cf.y, x1, cf.w), acc[r]);
           }
           __syncwarp();
           if (lane == 0) mbar_arrive(empty + st);
           if (++st == n_stages) { st = 0; ph ^= 1u; }
         }
         if (!ok) break;
-        dll_s[buf * 128 + row] = acc + gc;
+        dll_s[buf * 128 + gt] = warp_transpose_sum(acc) + gc;
         mbar_arrive(g_full + buf);
       }
     }
@@ -666,7 +826,7 @@ __host__ __device__ inline size_t f32_smem_floats(const Dims& dm) {
   const int E16 = round_up(dm.E, 16);
   const int dpad = round_up(dm.d, 32);
   return 128 * 33 + static_cast<size_t>(dm.E) * 33 + 128 * static_cast<size_t>(E16 + 1) + 2 * dpad +
-         epi_smem_floats(dm.K) + 128 + 24;
+         epi_smem_floats(dm.K) + 128;
 }
 
 template <bool kGauss, int KM>
@@ -684,11 +844,9 @@ k_router_fwd_f32(const FwdParams p) {
   float* gb = ga + dpad;                   // [dpad]
   float* epi = gb + dpad;                  // epilogue tables
   float* dll_s = epi + epi_smem_floats(dm.K);   // [128]
-  float* red = dll_s + 128;                // [17]
   uint64_t* bars = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(red + 17) + 7) & ~uintptr_t(7));   // [2]
+      (reinterpret_cast<uintptr_t>(dll_s + 128) + 7) & ~uintptr_t(7));   // [2]
   int* abort_flag = reinterpret_cast<int*>(bars + 2);
-  int* s_bin = abort_flag + 1;
 
   const int t = threadIdx.x, r = t >> 2, qd = t & 3;
   const int tile = blockIdx.x;
@@ -699,9 +857,14 @@ k_router_fwd_f32(const FwdParams p) {
     mbar_init(bars + 1, 128);
     fence_mbar_init();
   }
-  for (int e = t; e < E; e += 512) s_bin[e] = p.ws.expert_bin[e];
   float gc = 0.f;
-  if (kGauss) gc = gauss_coefficients(p.mu, p.var, d, dpad, ga, gb, red, p.ws.status);
+  if (kGauss) {
+    for (int i = t; i < dpad; i += 512) {
+      ga[i] = p.ws.gcoef[i];
+      gb[i] = p.ws.gcoef[p.ws.dcoef + i];
+    }
+    gc = gauss_gc(p.ws.gcoef, p.ws.dcoef);
+  }
   float acc[kF32MaxE / 4];
 #pragma unroll
   for (int i = 0; i < kF32MaxE / 4; ++i) acc[i] = 0.f;
@@ -741,64 +904,78 @@ k_router_fwd_f32(const FwdParams p) {
   if (qd == 0) dll_s[r] = gacc + gc;
   __syncthreads();
   if (t < 128) {
-    struct Prov {
+    struct Src {
       const float* z;
-      int ncols;
-      __device__ void load32(int c, float (&v)[32]) const {
+      int E;
+      __device__ void load16(int c, float (&v)[16]) const {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = (32 * c + i < ncols) ? z[32 * c + i] : 0.f;
+        for (int i = 0; i < 16; ++i) v[i] = (16 * c + i < E) ? z[16 * c + i] : -FLT_MAX;
       }
-    } prov{zs + t * (E16 + 1), E16};
+    } src{zs + t * (E16 + 1), E};
     struct Rel {
       __device__ void operator()() const {}
     } rel;
     WaitCtx wc{abort_flag, p.ws.status, p.limit_ns};
-    EpiSmem es{epi, epi + 2 * dm.K * kPsStride, bars + 0, bars + 1, s_bin};
-    epilogue_tile<KM>(p, prov, rel, tile, t, t, 0, kGauss ? dll_s[t] : 0.f, es, wc);
+    const EpiSmem es = epi_smem(epi, dm.K, bars + 0, bars + 1);
+    uint32_t n_in = 0;
+    const TileMeta meta = load_tile_meta(p, tile, t);
+    epilogue_tile<KM>(p, src, rel, tile, t, 0, kGauss ? dll_s[t] : 0.f, meta, es, wc, n_in);
   }
 }
 
-template <bool kGauss>
-cudaError_t launch_tc(const FwdParams& p, const CUtensorMap& tmX, const CUtensorMap& tmW, int grid,
-                      int threads, size_t smem, int N, int n_stages, cudaStream_t s) {
-  auto k = (p.dm.k <= 8) ? k_router_fwd_tc<kGauss, 8> : k_router_fwd_tc<kGauss, 16>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  k<<<grid, threads, smem, s>>>(tmX, tmW, p, N, n_stages);
-  return cudaGetLastError();
-}
-
-template <bool kGauss>
-cudaError_t launch_f32(const FwdParams& p, size_t smem, cudaStream_t s) {
-  auto k = (p.dm.k <= 8) ? k_router_fwd_f32<kGauss, 8> : k_router_fwd_f32<kGauss, 16>;
-  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  k<<<p.n_tiles, 512, smem, s>>>(p);
-  return cudaGetLastError();
+// Top-k insertion width: k rounded up to 2, 4, 6, 8 or 16.
+template <class F>
+cudaError_t dispatch_km(int k, F&& f) {
+  if (k <= 2) return f(std::integral_constant<int, 2>());
+  if (k <= 4) return f(std::integral_constant<int, 4>());
+  if (k <= 6) return f(std::integral_constant<int, 6>());
+  if (k <= 8) return f(std::integral_constant<int, 8>());
+  return f(std::integral_constant<int, 16>());
 }
 
 }  // namespace
 
 cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
-                                   const CUtensorMap& tmW, int n_sms, cudaStream_t s) {
+                                   const CUtensorMap& tmW, const CUtensorMap* tmG, int n_sms,
+                                   cudaStream_t s) {
   const int N = round_up(p.dm.E, 16);
   const bool gauss = p.M_in == nullptr;
-  // as many pipeline stages as fit next to the epilogue's shared memory
-  int n_stages = 8;
-  while (n_stages > 2 && fwd_smem_bytes(N, n_stages, p.dm.d, p.dm.K, p.dm.E, gauss) > 227u * 1024u)
-    --n_stages;
-  const size_t smem = fwd_smem_bytes(N, n_stages, p.dm.d, p.dm.K, p.dm.E, gauss);
+  // as many pipeline stages as fit next to the epilogue's shared memory; the scores are staged
+  // for a coalesced store when that still leaves five stages
+  auto stages_for = [&](bool stg) {
+    int n = 8;
+    while (n > 2 && fwd_smem_bytes(N, n, p.dm.d, p.dm.K, p.dm.E, gauss, stg) > 227u * 1024u) --n;
+    return n;
+  };
+  const bool use_stg = tmG != nullptr && stages_for(true) >= 5;
+  const int n_stages = stages_for(use_stg);
+  const size_t smem = fwd_smem_bytes(N, n_stages, p.dm.d, p.dm.K, p.dm.E, gauss, use_stg);
   if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
   const int grid = p.n_tiles < n_sms ? p.n_tiles : n_sms;
-  return gauss ? launch_tc<true>(p, tmX, tmW, grid, 320, smem, N, n_stages, s)
-               : launch_tc<false>(p, tmX, tmW, grid, 192, smem, N, n_stages, s);
+  const CUtensorMap& tg = use_stg ? *tmG : tmX;           // unused without staging
+  return dispatch_km(p.dm.k, [&](auto km) -> cudaError_t {
+    constexpr int KM = decltype(km)::value;
+    auto k = gauss ? k_router_fwd_tc<true, KM> : k_router_fwd_tc<false, KM>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k<<<grid, gauss ? 320 : 192, smem, s>>>(tmX, tmW, tg, p, N, n_stages, use_stg ? 1 : 0);
+    return cudaGetLastError();
+  });
 }
 
 cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s) {
   if (p.dm.E > kF32MaxE) return cudaErrorInvalidValue;
   const size_t smem = sizeof(float) * f32_smem_floats(p.dm) + sizeof(int) * round_up(p.dm.E, 4) + 64;
   if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
-  return (p.M_in == nullptr) ? launch_f32<true>(p, smem, s) : launch_f32<false>(p, smem, s);
+  const bool gauss = p.M_in == nullptr;
+  return dispatch_km(p.dm.k, [&](auto km) -> cudaError_t {
+    constexpr int KM = decltype(km)::value;
+    auto k = gauss ? k_router_fwd_f32<true, KM> : k_router_fwd_f32<false, KM>;
+    cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k<<<p.n_tiles, 512, smem, s>>>(p);
+    return cudaGetLastError();
+  });
 }
 
 }  // namespace smoes

@@ -44,15 +44,18 @@ struct WsView {
   float* gsave;              // [T * E] softmax scores saved by the forward
   float* dw_part;            // [G * E * d] per-token-group partial dW
   uint8_t* dz_img;           // [ceil(T/64)][hi|lo][E_pad/64][64 rows][128 B] dz in the MMA layout
-  int32_t* perm_scratch;     // permutation block counts / offsets
+  int32_t* perm_scratch;     // permutation block counts [n_blocks * K]
   uint32_t* attn_ticket;     // [B * ceil(S/128)] head tickets of the attention score
   float* attn_part;          // [H_max * T] per-head vision mass
+  float* gcoef;              // Gaussian score coefficients: ga[dcoef], gb[dcoef], part[dcoef/256]
+  int dcoef;                 // round_up(d, 256)
 };
 
 struct Dims {
   int T, d, E, k, K, B, N_B, renorm;
   int pstride;               // piece_stride(K)
   int n_groups;              // ceil(T / 128): forward tiles = partial-sum groups
+  int contig_bins;           // bin b holds experts [b N_B, (b+1) N_B) and N_B % 4 == 0
 };
 
 struct FwdParams {
@@ -107,18 +110,19 @@ struct PermParams {
   uint32_t* perm_mask;
   int32_t* dispatch;
   int32_t* expert_counts;
-  int32_t* blk_counts;       // [n_blocks * K]
-  int32_t* blk_offsets;      // [n_blocks * K]
+  int32_t* blk_counts;       // [n_blocks * K] pair counts per block and bin
+  uint32_t* sync;            // [2] grid barrier: arrivals, generation (zero between calls)
   uint32_t* status;
   int n_blocks;
   int rounds;                // 256-token rounds per block
+  uint64_t limit_ns;
 };
 
 struct GaussParams {
   int T, d;
   const void* X;
-  const float* mu;
-  const float* var;
+  const float* gcoef;        // written by the coefficient kernel launched just before
+  int dcoef;
   float inv_tau;
   float* M;
   uint32_t* status;
@@ -150,17 +154,20 @@ struct AttnParams {
 constexpr int kStaticPermBlocks = 1024;
 struct StaticPermScratch {
   int32_t blk_counts[kStaticPermBlocks * kMaxBins];
-  int32_t blk_offsets[kStaticPermBlocks * kMaxBins];
   int32_t expert_bin[kMaxExperts];
   int32_t expert_slot[kMaxExperts];
   uint32_t status[4];
+  uint32_t sync[4];
 };
 // Device address of that array on the current device (resolved once per device).
 cudaError_t static_perm_scratch(StaticPermScratch** out);
 
 // ------------------------------------------------------------------ launchers (in .cu files)
+// tmG: TMA map of the saved softmax scores [T, E] fp32 (box 32 x 128, 128-byte swizzle), or
+// null to store them row by row.
 cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
-                                   const CUtensorMap& tmW, int n_sms, cudaStream_t s);
+                                   const CUtensorMap& tmW, const CUtensorMap* tmG, int n_sms,
+                                   cudaStream_t s);
 cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s);
 cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX,
                                    const CUtensorMap& tmW, const CUtensorMap& tmDX,
@@ -170,6 +177,9 @@ cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s);
 cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s);
 cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s);
 cudaError_t launch_gauss_score(const GaussParams& p, smoes_dtype dt, int n_sms, cudaStream_t s);
+// Coefficients of the Gaussian log-likelihood difference (eq. 8) into coef = ga | gb | part.
+cudaError_t launch_gauss_coef(const float* mu, const float* var, int d, int dcoef, float* coef,
+                              uint32_t* status, cudaStream_t s);
 cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                              int n_sms, cudaStream_t s);
 
