@@ -10,8 +10,8 @@
 #include "smoes_internal.cuh"
 
 namespace smoes {
-int perm_blocks(int T);
-int perm_rounds(int T);
+int perm_blocks(int T, int k);
+int perm_rounds(int T, int k);
 }
 
 using namespace smoes;
@@ -261,7 +261,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
     P->bwd_slices = 1;
     P->bwd_groups = std::max(1, P->bwd_tiles);
   }
-  P->perm_nblocks = std::max(1, perm_blocks(T));
+  P->perm_nblocks = std::max(1, perm_blocks(T, d.k));
 
   // workspace layout
   Layout& L = P->L;
@@ -554,7 +554,7 @@ smoes_status smoes_bin_permute(smoes_plan P, const int32_t* topk_idx, const int3
   p.sync = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + P->L.perm_sync);
   p.status = v.status;
   p.n_blocks = P->perm_nblocks;
-  p.rounds = perm_rounds(d.T);
+  p.rounds = perm_rounds(d.T, d.k);
   p.limit_ns = kWaitLimitNs;
   return cuda_status(launch_bin_permute(p, stream));
 }
@@ -610,7 +610,7 @@ extern "C" smoes_status smoes_bin_permute_noalloc(smoes_plan P, const int32_t* t
   p.sync = sp->sync;
   p.status = sp->status;
   p.n_blocks = P->perm_nblocks;
-  p.rounds = perm_rounds(d.T);
+  p.rounds = perm_rounds(d.T, d.k);
   p.limit_ns = kWaitLimitNs;
   return cuda_status(launch_bin_permute(p, stream));
 }

@@ -21,25 +21,36 @@ namespace {
 constexpr int kPermThreads = 256;                    // one token per thread and round
 constexpr int kPermWarps = kPermThreads / 32;
 
+// One token's selection: its chosen experts (-1 for none) with their bins and slot bits, the
+// set of the bins and the token's modality (0 vision, 1 text). KM >= k, a compile-time bound
+// that keeps the arrays in registers.
+template <int KM>
 struct TokenSel {
-  int e[kMaxTopK];
-  int b[kMaxTopK];
+  int e[KM];
+  int b[KM];
+  uint32_t sbit[KM];
   uint32_t bins;
+  int m;
 };
 
-__device__ __forceinline__ void load_sel(const PermParams& p, const int* s_bin, int j, TokenSel& s) {
+template <int KM>
+__device__ __forceinline__ void load_sel(const PermParams& p, const int* s_bin, const int* s_slot,
+                                         int j, TokenSel<KM>& s) {
   s.bins = 0u;
-  int e[kMaxTopK];
+  int e[KM];
 #pragma unroll
-  for (int i = 0; i < kMaxTopK; ++i) e[i] = i < p.k ? p.topk_idx[static_cast<size_t>(j) * p.k + i] : -1;
+  for (int i = 0; i < KM; ++i) e[i] = i < p.k ? p.topk_idx[static_cast<size_t>(j) * p.k + i] : -1;
+  s.m = (p.is_vision && !p.is_vision[j]) ? 1 : 0;
 #pragma unroll
-  for (int i = 0; i < kMaxTopK; ++i) {
+  for (int i = 0; i < KM; ++i) {
     s.e[i] = -1;
     s.b[i] = -1;
+    s.sbit[i] = 0u;
     if (i < p.k) {
       if (e[i] >= 0 && e[i] < p.E) {
         s.e[i] = e[i];
         s.b[i] = s_bin[e[i]];
+        s.sbit[i] = 1u << s_slot[e[i]];
         s.bins |= 1u << s.b[i];
       } else {
         atomicOr(p.status, kStatusData);
@@ -68,12 +79,12 @@ __device__ bool grid_barrier(uint32_t* sync, uint32_t n, uint64_t limit_ns, uint
       atomicOr(status, kStatusTimeout);
       return false;
     }
-    __nanosleep(64);
   }
   __threadfence();
   return true;
 }
 
+template <int KM>
 __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
   __shared__ int s_bin[kMaxExperts];
   __shared__ int s_slot[kMaxExperts];
@@ -93,13 +104,19 @@ __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
   for (int i = threadIdx.x; i < 2 * p.E; i += kPermThreads) ecnt[i] = 0;
   __syncthreads();
 
-  // count: lane kb of each warp accumulates the warp's pairs in bin kb
+  // count: lane kb of each warp accumulates the warp's pairs in bin kb; the first round's
+  // selections stay in registers for the scatter
   int cnt = 0;
+  TokenSel<KM> s0;
+  s0.bins = 0u;
+  s0.m = 0;
   for (int r = 0; r < p.rounds; ++r) {
     const int j = (blockIdx.x * p.rounds + r) * kPermThreads + threadIdx.x;
-    TokenSel s;
+    TokenSel<KM> s;
     s.bins = 0u;
-    if (j < p.T) load_sel(p, s_bin, j, s);
+    s.m = 0;
+    if (j < p.T) load_sel<KM>(p, s_bin, s_slot, j, s);
+    if (r == 0) s0 = s;
     for (int kb = 0; kb < K; ++kb) {
       const int c = __popc(__ballot_sync(0xffffffffu, (s.bins >> kb) & 1u));
       if (lane == kb) cnt += c;
@@ -110,7 +127,7 @@ __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
   if (threadIdx.x < K) {
     int t = 0;
     for (int w = 0; w < kPermWarps; ++w) t += wcnt[w][threadIdx.x];
-    p.blk_counts[blockIdx.x * K + threadIdx.x] = t;
+    p.blk_counts[threadIdx.x * p.n_blocks + blockIdx.x] = t;     // bin-major
   }
   if (blockIdx.x == 0) {
     for (int i = threadIdx.x; i < K * K; i += kPermThreads) p.dispatch[i] = 0;
@@ -122,13 +139,20 @@ __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
   __syncthreads();
   if (!ok_s) return;
 
-  // offsets: warp w sums bins w, w + 8, ... over all blocks (lanes stride the blocks)
+  // offsets: warp w sums bins w, w + 8, ... over all blocks (lanes stride the blocks, eight
+  // loads in flight per lane and round)
   for (int kb = warp; kb < K; kb += kPermWarps) {
     int pre = 0, tot = 0;
-    for (int b = lane; b < p.n_blocks; b += 32) {
-      const int c = __ldcg(p.blk_counts + b * K + kb);
-      tot += c;
-      if (b < static_cast<int>(blockIdx.x)) pre += c;
+    const int* row = p.blk_counts + kb * p.n_blocks;
+    for (int b0 = lane; b0 < p.n_blocks; b0 += 8 * 32) {
+      int c[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) c[u] = b0 + 32 * u < p.n_blocks ? __ldcg(row + b0 + 32 * u) : 0;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        tot += c[u];
+        if (b0 + 32 * u < static_cast<int>(blockIdx.x)) pre += c[u];
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -157,9 +181,14 @@ __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
   for (int r = 0; r < p.rounds; ++r) {
     const int j = (blockIdx.x * p.rounds + r) * kPermThreads + threadIdx.x;
     const bool valid = j < p.T;
-    TokenSel s;
+    TokenSel<KM> s;
     s.bins = 0u;
-    if (valid) load_sel(p, s_bin, j, s);
+    s.m = 0;
+    if (r == 0) {
+      s = s0;
+    } else if (valid) {
+      load_sel<KM>(p, s_bin, s_slot, j, s);
+    }
     int home = 0;
     if (valid) {
       home = p.home ? p.home[j] : static_cast<int>((static_cast<long long>(j) * K) / p.T);
@@ -183,24 +212,25 @@ __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
       base[threadIdx.x] = run;                          // carried into the next round
     }
     __syncthreads();
+    // lanes with the same dispatch home add their pairs with one atomic per (warp, bin, home)
+    const unsigned same_home = __match_any_sync(0xffffffffu, home);
     for (int kb = 0; kb < K; ++kb) {
       const unsigned bal = __ballot_sync(0xffffffffu, (s.bins >> kb) & 1u);
       if ((s.bins >> kb) & 1u) {
         const int pos = wcnt[warp][kb] + __popc(bal & lt_mask);
         uint32_t mask = 0u;
 #pragma unroll
-        for (int i = 0; i < kMaxTopK; ++i)
-          if (i < p.k && s.b[i] == kb) mask |= 1u << s_slot[s.e[i]];
+        for (int i = 0; i < KM; ++i) mask |= (s.b[i] == kb) ? s.sbit[i] : 0u;
         p.perm_token[pos] = j;
         p.perm_mask[pos] = mask;
-        if (home >= 0) atomicAdd(&disp[home * K + kb], 1);
+        const unsigned grp = bal & same_home;
+        if (home >= 0 && lane == __ffs(grp) - 1) atomicAdd(&disp[home * K + kb], __popc(grp));
       }
     }
     if (valid && p.expert_counts) {
-      const int m = p.is_vision[j] ? 0 : 1;
 #pragma unroll
-      for (int i = 0; i < kMaxTopK; ++i)
-        if (i < p.k && s.e[i] >= 0) atomicAdd(&ecnt[m * p.E + s.e[i]], 1);
+      for (int i = 0; i < KM; ++i)
+        if (s.e[i] >= 0) atomicAdd(&ecnt[s.m * p.E + s.e[i]], 1);
     }
     __syncthreads();                                    // wcnt reused by the next round
   }
@@ -237,35 +267,47 @@ cudaError_t static_perm_scratch(StaticPermScratch** out) {
   return cudaSuccess;
 }
 
+template <class F>
+cudaError_t with_kernel(int k, F&& f) {
+  if (k <= 2) return f(k_perm<2>);
+  if (k <= 4) return f(k_perm<4>);
+  if (k <= 6) return f(k_perm<6>);
+  if (k <= 8) return f(k_perm<8>);
+  return f(k_perm<16>);
+}
+
 // Blocks of the permutation: all must be resident at once (the grid barrier), and at most
 // kStaticPermBlocks. Rounds of 256 tokens per block grow once the batch needs more blocks.
-int perm_max_blocks() {
+int perm_max_blocks(int k) {
   static std::mutex mu;
-  static int cached[64] = {};
+  static int cached[64][5] = {};
+  const int v = k <= 2 ? 0 : k <= 4 ? 1 : k <= 6 ? 2 : k <= 8 ? 3 : 4;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
   std::lock_guard<std::mutex> lock(mu);
-  if (cached[dev] == 0) {
+  if (cached[dev][v] == 0) {
     int sms = 0, per_sm = 0;
-    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_perm, kPermThreads, 0) != cudaSuccess)
-      return 1;
-    cached[dev] = std::max(1, std::min(kStaticPermBlocks, sms * per_sm));
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
+    const cudaError_t e = with_kernel(k, [&](auto kern) {
+      return cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kPermThreads, 0);
+    });
+    if (e != cudaSuccess) return 1;
+    cached[dev][v] = std::max(1, std::min(kStaticPermBlocks, sms * per_sm));
   }
-  return cached[dev];
+  return cached[dev][v];
 }
-int perm_rounds(int T) {
+int perm_rounds(int T, int k) {
   const int units = (T + kPermThreads - 1) / kPermThreads;
-  const int cap = perm_max_blocks();
+  const int cap = perm_max_blocks(k);
   return units <= cap ? 1 : (units + cap - 1) / cap;
 }
-int perm_blocks(int T) {
-  const int per = kPermThreads * perm_rounds(T);
+int perm_blocks(int T, int k) {
+  const int per = kPermThreads * perm_rounds(T, k);
   return (T + per - 1) / per;
 }
 
 cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s) {
-  if (p.n_blocks > perm_max_blocks()) return cudaErrorInvalidValue;
+  if (p.n_blocks > perm_max_blocks(p.k)) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(p.n_blocks);
   cfg.blockDim = dim3(kPermThreads);
@@ -275,7 +317,7 @@ cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s) {
   attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_perm, p);
+  return with_kernel(p.k, [&](auto kern) { return cudaLaunchKernelEx(&cfg, kern, p); });
 }
 
 }  // namespace smoes
