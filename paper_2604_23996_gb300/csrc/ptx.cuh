@@ -85,6 +85,31 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const 
   }
 }
 
+// Grid barrier for co-resident blocks, called by one thread per block. sync[0] counts
+// arrivals, sync[1] is the generation; the last block resets the count and advances the
+// generation, so the pair is zero-count again between calls. A wait that exceeds limit_ns sets
+// the timeout status and returns false.
+__device__ inline bool grid_barrier(uint32_t* sync, uint32_t n, uint64_t limit_ns, uint32_t* status) {
+  volatile uint32_t* gen = sync + 1;
+  const uint32_t g0 = *gen;
+  __threadfence();
+  if (atomicAdd(sync, 1u) == n - 1) {
+    atomicExch(sync, 0u);
+    __threadfence();
+    atomicAdd(sync + 1, 1u);
+    return true;
+  }
+  const uint64_t t0 = global_ns();
+  while (*gen == g0) {
+    if (global_ns() - t0 > limit_ns) {
+      atomicOr(status, 2u);   // the timeout status bit
+      return false;
+    }
+  }
+  __threadfence();
+  return true;
+}
+
 // ---------------------------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");

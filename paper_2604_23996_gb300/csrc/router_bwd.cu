@@ -84,7 +84,11 @@ __device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
 
 // ------------------------------------------------------------------ dz preparation (bf16 path)
 // TPT = E_pad/8 threads per token, 8 experts each; the token's sum over experts is a shuffle
-// reduction inside its TPT-lane group. Rows beyond T and padded experts are written as zeros.
+// reduction inside its TPT-lane group. dz is written as the bf16 hi/lo pair (dz = hi + lo to
+// ~2^-17 relative) in the 128-byte-swizzled operand image of its 64-token tile,
+// [tile][hi | lo][E_pad/64][64 rows][128 B], which the main kernel bulk-copies. Rows beyond T and
+// padded experts are zeros. With consecutive bins of a multiple of 4 experts, a thread's 8
+// experts lie in at most two bins: their coefficients are read once per bin.
 template <int TPT>
 __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
   const Dims& dm = p.dm;
@@ -97,7 +101,6 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
   if (j >= n_rows) return;                            // whole TPT groups exit together
   const bool valid = j < dm.T;
   float g[8], u[8];
-  float dv = 0.f, dt = 0.f;
   if (valid) {
     const float* grow = p.ws.gsave + static_cast<size_t>(j) * E;
     if ((E & 3) == 0 && e0 + 8 <= E) {
@@ -109,16 +112,23 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
       for (int q = 0; q < 8; ++q) g[q] = (e0 + q < E) ? __ldcg(grow + e0 + q) : 0.f;
     }
     const float2 m = __ldg(reinterpret_cast<const float2*>(p.M) + j);
-    dv = m.x - 0.5f;
-    dt = m.y - 0.5f;
+    const float dv = m.x - 0.5f, dt = m.y - 0.5f;
     // the sample's coefficient table was written by the forward kernel and is read-only here
     const float* tb = p.ws.tabs + static_cast<size_t>(__ldg(p.ws.token_sample + j)) * 3 * K;
+    if (dm.contig_bins && e0 + 8 <= E) {
+      const int b0 = e0 / dm.N_B, b1 = (e0 + 7) / dm.N_B;
+      const float u0 = __ldg(tb + 2 * K + b0) + dv * __ldg(tb + b0) + dt * __ldg(tb + K + b0);
+      const float u1 = __ldg(tb + 2 * K + b1) + dv * __ldg(tb + b1) + dt * __ldg(tb + K + b1);
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      u[q] = 0.f;
-      if (e0 + q < E) {
-        const int b = __ldg(p.ws.expert_bin + e0 + q);
-        u[q] = __ldg(tb + 2 * K + b) + dv * __ldg(tb + b) + dt * __ldg(tb + K + b);
+      for (int q = 0; q < 8; ++q) u[q] = (e0 + q) / dm.N_B == b0 ? u0 : u1;
+    } else {
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        u[q] = 0.f;
+        if (e0 + q < E) {
+          const int b = __ldg(p.ws.expert_bin + e0 + q);
+          u[q] = __ldg(tb + 2 * K + b) + dv * __ldg(tb + b) + dt * __ldg(tb + K + b);
+        }
       }
     }
   } else {
@@ -178,11 +188,13 @@ __host__ __device__ inline BwdLayout bwd_layout(int E_pad, int n_xst) {
   L.dz = o;   o += 2u * 2u * static_cast<uint32_t>(E_pad) * 128u;   // 2 buffers x (hi, lo)
   L.xst = o;  o += static_cast<uint32_t>(n_xst) * 16384u;          // X stages [2 atoms][64][128 B]
   L.stg = o;  o += 2u * 16384u;                                    // dX staging [64][128] bf16 x2
-  L.bars = o; o += 8u * (2u * n_xst + 16u) + 16u;
+  L.bars = o; o += 8u * (2u * n_xst + 18u) + 16u;
   L.total = o + 1024u;
   return L;
 }
 
+// Roles (192 threads): warp 0 TMA / bulk-copy producer, warp 1 MMA issuer, warps 2-5 dX drain
+// and dW^T drain. After the last tile every CTA writes its dW^T partial; k_dw_reduce sums them.
 template <int E_pad>
 __global__ void __launch_bounds__(192, 1)
 k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
@@ -198,8 +210,8 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
   uint64_t* xfull = bars;
   uint64_t* xempty = bars + n_xst;
-  uint64_t* dz_full = bars + 2 * n_xst;       // [2]
-  uint64_t* dz_empty = dz_full + 2;           // [2]
+  uint64_t* dz_full = bars + 2 * n_xst;       // [2] the tile's dz image has landed
+  uint64_t* dz_empty = dz_full + 2;           // [2] the tile's MMAs have read it
   uint64_t* dx_full = dz_full + 4;            // [2]
   uint64_t* dx_empty = dz_full + 6;           // [2]
   uint64_t* wfull = dz_full + 8;
@@ -207,7 +219,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   uint64_t* drain = dz_full + 10;
   uint64_t* stg_free = dz_full + 11;          // [2] staging buffer may be rewritten
   uint64_t* stg_full = dz_full + 13;          // [2] staging buffer written
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dz_full + 16);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dz_full + 18);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -250,7 +262,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   const uint32_t tm_dx = tmem + 256u;          // two 64-column dX^T buffers after the dW^T blocks
 
   if (warp == 0) {
-    // -------------------------------------------------------------- TMA / bulk-copy producer
+    // -------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
       mbar_arrive_expect_tx(wfull, static_cast<uint32_t>(nb) * 2u * dz_half);
@@ -568,6 +580,16 @@ __global__ void __launch_bounds__(kDwSlices * kDwCols) k_dw_reduce(const BwdPara
 
 }  // namespace
 
+cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s) {
+  const int E_pad = round_up(p.dm.E, 64);
+  const long threads = static_cast<long>(p.n_tiles) * kBwdBT * (E_pad / 8);
+  const int blocks = static_cast<int>((threads + 255) / 256);
+  if (E_pad == 64) k_dz_prep<8><<<blocks, 256, 0, s>>>(p);
+  else if (E_pad == 128) k_dz_prep<16><<<blocks, 256, 0, s>>>(p);
+  else return cudaErrorInvalidValue;
+  return cudaGetLastError();
+}
+
 cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, const CUtensorMap& tmW,
                                    const CUtensorMap& tmDX, cudaStream_t s) {
   const int E_pad = round_up(p.dm.E, 64);
@@ -583,15 +605,6 @@ cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, c
   return cudaGetLastError();
 }
 
-cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s) {
-  const int E_pad = round_up(p.dm.E, 64);
-  const long threads = static_cast<long>(p.n_tiles) * kBwdBT * (E_pad / 8);
-  const int blocks = static_cast<int>((threads + 255) / 256);
-  if (E_pad == 64) k_dz_prep<8><<<blocks, 256, 0, s>>>(p);
-  else if (E_pad == 128) k_dz_prep<16><<<blocks, 256, 0, s>>>(p);
-  else return cudaErrorInvalidValue;
-  return cudaGetLastError();
-}
 
 cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s) {
   if (p.dm.E > kF32MaxE) return cudaErrorInvalidValue;
