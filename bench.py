@@ -221,11 +221,30 @@ def run_reference(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def rank_env():
+    """(rank, world size, local rank) of this process as torchrun sets them (1 process: 0, 1, 0)."""
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def max_over_ranks(x, world, device):
+    """The largest value of x over all ranks (the job's time is its slowest replica's)."""
+    if world <= 1:
+        return float(x)
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(tokens_per_replica, world, ms):
+    """Whole-job tokens/s: every replica processes tokens_per_replica in ms milliseconds."""
+    return world * tokens_per_replica / (ms * 1e-3)
+
+
 def main():
     args = parse()
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    rank, world, local = rank_env()
     if args.impl == "reference":
         run_reference(args, rank, world)
         return
@@ -337,13 +356,9 @@ def main():
     t_step = [e[0].elapsed_time(e[-1]) for e in evs]
     t_part = {name: [e[i].elapsed_time(e[i + 1]) for e in evs] for i, (name, _) in enumerate(parts)}
     t_bwd = t_part["bwd"]
-    total_ms = float(np.sum(t_step))
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(float(np.sum(t_step)), world, dev)
     ms_per_step = total_ms / args.steps
-    value = world * wl.T / (ms_per_step * 1e-3)
+    value = job_rate(wl.T, world, ms_per_step)
 
     # end to end through the public API: host inputs in pinned memory, copies inside the region
     e2e = None
@@ -385,7 +400,8 @@ def main():
             b.record()
             b.synchronize()
             t_e2e += a.elapsed_time(b)
-        e2e = {"value": world * wl.T / (t_e2e / args.steps * 1e-3), "unit": UNIT,
+        t_e2e = max_over_ranks(t_e2e, world, dev)
+        e2e = {"value": job_rate(wl.T, world, t_e2e / args.steps), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
     if rank != 0:
