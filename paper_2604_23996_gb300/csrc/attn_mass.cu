@@ -2,14 +2,17 @@
 //
 // For sequence b and query j:  Mtilde_v[b,j] = (1/H) sum_h sum_{j'} softmax_{j'}(s q_j.k_j' + beta_j') m_j',
 // the head-averaged attention matrix applied to the keys' carried vision score m (eq. 3; the hard
-// labels of eq. 2 at layer 0). As the paper notes, this equals attention with the score as the
-// value vector, so it runs FlashAttention-style without materialising the attention matrix:
-// per (sequence, head, 128-query tile) the scores S = Q K^T of each 128-key block are formed on
-// tcgen05 tensor cores (TMA-fed, accumulator in TMEM); four softmax warps (one query row per
-// thread) keep the online max, the normaliser l = sum e^(s - max) and the vision mass
-// a = sum e^(s - max) m_j'. The head's score a / l goes to the workspace; the last head of each
-// (sequence, query tile) to finish averages the heads in fixed order and writes M (optionally
-// blended with the carried score by eq. 4).
+// labels of eq. 2 at layer 0). This equals attention with the score as the value vector, so it
+// runs FlashAttention-style without materialising the attention matrix.
+//
+// A work item is (sequence, head, pair of adjacent 128-query tiles). The two tiles share one
+// stream of 128-key blocks: for each block the tensor cores form S = Q K^T of both tiles
+// (tcgen05, TMA-fed, accumulators in TMEM, two buffers per tile). Two softmax groups of four
+// warps (one query row per thread, one group per tile) keep the online max, the normaliser
+// l = sum e^(s - max) and the vision mass a = sum e^(s - max) m_j'. The head's score a / l goes
+// to the workspace; the last head of each (sequence, query tile) to finish averages the heads in
+// fixed order and writes M (optionally blended with the carried score by eq. 4). Items are
+// handed out longest first so that the CTAs finish together.
 #include <cuda_bf16.h>
 #include <math_constants.h>
 
@@ -31,30 +34,66 @@ struct AttnLayout {
 __host__ __device__ inline AttnLayout attn_layout(int n_ks) {
   AttnLayout L;
   uint32_t o = 0;
-  L.q = o;    o += kTile;                                  // Q tile [2 atoms][128 rows][128 B]
+  L.q = o;    o += 2u * kTile;                             // two Q tiles [2 atoms][128 rows][128 B]
   L.k = o;    o += static_cast<uint32_t>(n_ks) * kTile;    // K blocks
-  L.mk = o;   o += 2u * kAT * 8u;                          // (bias*log2e, m) per key, 2 buffers
-  L.bars = o; o += 8u * (2u * n_ks + 12u) + 16u;
+  L.mk = o;   o += 2u * 2u * 2u * kAT * 4u;                // bias*log2e [128] | m [128]: group x buffer
+  L.bars = o; o += 8u * (2u * n_ks + 24u) + 32u;
   L.total = o + 1024u;
   return L;
 }
 
-// Work item -> (sequence b, head h, query tile qt). Items are ordered head-major so that the
-// items running at the same time share keys in L2; a CTA's items cycle through tile sizes.
-__device__ __forceinline__ void decode_item(const AttnParams& p, int item, int& b, int& h, int& qt) {
-  const int bh = item / p.n_qtiles;
-  qt = item - bh * p.n_qtiles;
-  b = bh / p.H;
-  h = bh - b * p.H;
+// 2^x on the special-function unit (flushes results below 2^-126 to zero).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
+// Packed fp32 pair arithmetic (one instruction for two lanes' worth of work per thread):
+// (d0, d1) = (a0, a1) * (b0, b1) + (c0, c1), and (d0, d1) = (a0, a1) + (b0, b1).
+__device__ __forceinline__ void fma2(float& d0, float& d1, float a0, float a1, float b0, float b1,
+                                     float c0, float c1) {
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\t"
+      "mov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+__device__ __forceinline__ void add2(float& d0, float& d1, float a0, float a1, float b0, float b1) {
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "add.rn.f32x2 rd, ra, rb;\n\t"
+      "mov.b64 {%0, %1}, rd;\n\t}"
+      : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
+// Work item -> (sequence b, head h, query-tile pair pr). Pairs run longest (last) first; within
+// a pair index the heads of all sequences follow each other, so concurrent items share L2 keys.
+struct Item {
+  int b, h, qt0, nq;          // first query tile, tiles in the pair (1 or 2)
+};
+
+__device__ __forceinline__ Item decode_item(const AttnParams& p, int item) {
+  const int n_pairs = (p.n_qtiles + 1) / 2;
+  const int BH = p.B * p.H;
+  const int pr = n_pairs - 1 - item / BH;
+  const int bh = item - (item / BH) * BH;
+  Item it;
+  it.b = bh / p.H;
+  it.h = bh - it.b * p.H;
+  it.qt0 = 2 * pr;
+  it.nq = min(2, p.n_qtiles - it.qt0);
+  return it;
+}
+
+// Key blocks query tile qt attends to.
 __device__ __forceinline__ int kblocks_of(const AttnParams& p, int qt) {
   const int nk = (p.S + kAT - 1) / kAT;
   return p.causal ? min(qt + 1, nk) : nk;
 }
 
 template <bool kFloatM>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(320, 1)
 k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
             const AttnParams p, const int n_ks) {
   extern __shared__ uint8_t smem_raw[];
@@ -62,23 +101,25 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   const AttnLayout L = attn_layout(n_ks);
   uint8_t* qs = base + L.q;
   uint8_t* ks = base + L.k;
-  float2* mk = reinterpret_cast<float2*>(base + L.mk);
+  float* mk = reinterpret_cast<float*>(base + L.mk);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
   uint64_t* kfull = bars;
   uint64_t* kempty = bars + n_ks;
-  uint64_t* q_full = bars + 2 * n_ks;
-  uint64_t* q_empty = q_full + 1;
-  uint64_t* s_full = q_full + 2;      // [2]
-  uint64_t* s_empty = q_full + 4;     // [2]
-  uint64_t* mk_bar = q_full + 6;      // [2] keys' (bias, m) staged by the softmax group
-  uint64_t* out_bar = q_full + 8;     // head results of the tile written
-  uint64_t* drain = q_full + 9;
-  uint64_t* dec_bar = q_full + 10;    // the ticket decision of the tile is published
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 12);
+  uint64_t* q_full = bars + 2 * n_ks;   // [2] per tile of the pair
+  uint64_t* q_empty = q_full + 2;       // [2]
+  uint64_t* s_full = q_full + 4;        // [tile][buf]
+  uint64_t* s_empty = q_full + 8;       // [tile][buf]
+  uint64_t* mk_bar = q_full + 12;       // [tile][buf] keys' (bias, m) staged by that group
+  uint64_t* out_bar = q_full + 16;      // [tile] head results of the tile written
+  uint64_t* dec_bar = q_full + 18;      // [tile] the ticket decision of the tile is published
+  uint64_t* drain = q_full + 20;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 22);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
-  volatile uint32_t* decision = reinterpret_cast<volatile uint32_t*>(tmem_slot + 2);
+  volatile uint32_t* decision = reinterpret_cast<volatile uint32_t*>(tmem_slot + 2);   // [2]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int BH = p.B * p.H;
+  const int n_items = ((p.n_qtiles + 1) / 2) * BH;
   WaitCtx wc{abort_flag, p.status, p.limit_ns};
   if (threadIdx.x == 0) {
     *abort_flag = 0;
@@ -86,21 +127,23 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       mbar_init(kfull + i, 1);
       mbar_init(kempty + i, 1);
     }
-    mbar_init(q_full, 1);
-    mbar_init(q_empty, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(s_full + i, 1);
-      mbar_init(s_empty + i, 128);
-      mbar_init(mk_bar + i, 128);
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(q_full + t, 1);
+      mbar_init(q_empty + t, 1);
+      mbar_init(out_bar + t, 128);
+      mbar_init(dec_bar + t, 1);
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(s_full + 2 * t + i, 1);
+        mbar_init(s_empty + 2 * t + i, 128);
+        mbar_init(mk_bar + 2 * t + i, 128);
+      }
     }
-    mbar_init(out_bar, 128);
-    mbar_init(dec_bar, 1);
     mbar_init(drain, 1);
     fence_mbar_init();
     tma_prefetch_desc(&tmQ);
     tma_prefetch_desc(&tmK);
   }
-  if (warp == 1) tmem_alloc(tmem_slot, 256);
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -111,19 +154,21 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     if (lane == 0) {
       int st = 0;
       uint32_t ph = 0;
-      int it = 0;
+      int nqt[2] = {0, 0};              // items that used Q buffer t: its barrier phase
       long issued = 0;
       bool ok = true;
-      for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++it) {
-        int b, h, qt;
-        decode_item(p, item, b, h, qt);
-        const int row0 = (b * p.H + h) * p.S;
-        if (!mbar_wait(q_empty, (static_cast<uint32_t>(it) & 1u) ^ 1u, wc)) { ok = false; break; }
-        mbar_arrive_expect_tx(q_full, kTile);
-        tma_load_2d(qs, &tmQ, q_full, 0, row0 + qt * kAT);
-        tma_load_2d(qs + kTile / 2, &tmQ, q_full, 64, row0 + qt * kAT);
-        const int nkb = kblocks_of(p, qt);
-        for (int kb = 0; kb < nkb; ++kb) {
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        const Item w = decode_item(p, item);
+        const int row0 = (w.b * p.H + w.h) * p.S;
+        for (int t = 0; t < w.nq && ok; ++t) {
+          if (!mbar_wait(q_empty + t, (static_cast<uint32_t>(nqt[t]) & 1u) ^ 1u, wc)) { ok = false; break; }
+          ++nqt[t];
+          mbar_arrive_expect_tx(q_full + t, kTile);
+          tma_load_2d(qs + t * kTile, &tmQ, q_full + t, 0, row0 + (w.qt0 + t) * kAT);
+          tma_load_2d(qs + t * kTile + kTile / 2, &tmQ, q_full + t, 64, row0 + (w.qt0 + t) * kAT);
+        }
+        const int nkb = kblocks_of(p, w.qt0 + w.nq - 1);
+        for (int kb = 0; kb < nkb && ok; ++kb) {
           if (!mbar_wait(kempty + st, ph ^ 1u, wc)) { ok = false; break; }
           uint8_t* kd = ks + st * kTile;
           mbar_arrive_expect_tx(kfull + st, kTile);
@@ -139,7 +184,8 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         wd.abort_flag = &dummy;
         for (long q = (issued > n_ks ? issued - n_ks : 0); q < issued; ++q)
           mbar_wait(kfull + (q % n_ks), static_cast<uint32_t>((q / n_ks) & 1), wd);
-        mbar_wait(q_full, static_cast<uint32_t>((it) & 1), wd);
+        for (int t = 0; t < 2; ++t)
+          if (nqt[t] > 0) mbar_wait(q_full + t, static_cast<uint32_t>(nqt[t] - 1) & 1u, wd);
       }
     }
   } else if (warp == 1) {
@@ -148,35 +194,45 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       const uint32_t idesc = idesc_bf16(kAT, kAT, false, false);
       int st = 0;
       uint32_t ph = 0;
-      int blk = 0;                      // running block count: selects the TMEM buffer
-      int it = 0;
+      int blk[2] = {0, 0};              // running block count per tile: selects its TMEM buffer
+      int nqt[2] = {0, 0};
       bool ok = true;
-      for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++it) {
-        int b, h, qt;
-        decode_item(p, item, b, h, qt);
-        if (!mbar_wait(q_full, static_cast<uint32_t>(it) & 1u, wc)) { ok = false; break; }
+      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+        const Item w = decode_item(p, item);
+        for (int t = 0; t < w.nq && ok; ++t)
+          if (!mbar_wait(q_full + t, static_cast<uint32_t>(nqt[t]++) & 1u, wc)) ok = false;
+        if (!ok) break;
         tc_fence_after();
-        const uint32_t qa = smem_u32(qs);
-        const int nkb = kblocks_of(p, qt);
-        for (int kb = 0; kb < nkb; ++kb, ++blk) {
-          const int buf = blk & 1;
-          if (!mbar_wait(s_empty + buf, (static_cast<uint32_t>(blk >> 1) & 1u) ^ 1u, wc)) { ok = false; break; }
+        const int nkb0 = kblocks_of(p, w.qt0), nkb = kblocks_of(p, w.qt0 + w.nq - 1);
+        for (int kb = 0; kb < nkb; ++kb) {
           if (!mbar_wait(kfull + st, ph, wc)) { ok = false; break; }
           tc_fence_after();
           const uint32_t kbase = smem_u32(ks + st * kTile);
-          const uint32_t d_tmem = tmem + static_cast<uint32_t>(buf * kAT);
+          for (int t = 0; t < w.nq; ++t) {
+            if (t == 0 && kb >= nkb0) continue;       // past the first tile's diagonal
+            const int buf = blk[t] & 1;
+            if (!mbar_wait(s_empty + 2 * t + buf, (static_cast<uint32_t>(blk[t] >> 1) & 1u) ^ 1u, wc)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t qa = smem_u32(qs + t * kTile);
+            const uint32_t d_tmem = tmem + static_cast<uint32_t>((2 * t + buf) * kAT);
 #pragma unroll
-          for (int kk = 0; kk < kHd / 16; ++kk) {
-            const uint32_t off = (kk >> 2) * (kTile / 2) + (kk & 3) * 32;
-            umma_bf16(d_tmem, sdesc_sw128(qa + off, 16, 1024), sdesc_sw128(kbase + off, 16, 1024), idesc,
-                      kk > 0 ? 1u : 0u);
+            for (int kk = 0; kk < kHd / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * (kTile / 2) + (kk & 3) * 32;
+              umma_bf16(d_tmem, sdesc_sw128(qa + off, 16, 1024), sdesc_sw128(kbase + off, 16, 1024), idesc,
+                        kk > 0 ? 1u : 0u);
+            }
+            umma_commit(s_full + 2 * t + buf);
+            ++blk[t];
           }
+          if (!ok) break;
           umma_commit(kempty + st);
-          umma_commit(s_full + buf);
           if (++st == n_ks) { st = 0; ph ^= 1u; }
         }
         if (!ok) break;
-        umma_commit(q_empty);           // the Q tile may be replaced once its MMAs are done
+        for (int t = 0; t < w.nq; ++t) umma_commit(q_empty + t);   // Q tiles may be replaced
       }
       umma_commit(drain);
       WaitCtx wd = wc;
@@ -185,90 +241,126 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       mbar_wait(drain, 0, wd);
     }
   } else {
-    // ---------------------------------------------------------------- softmax group (4 warps)
+    // ---------------------------------------------------------------- softmax groups (2 x 4 warps)
+    const int t = (warp - 2) >> 2;             // query tile of the pair handled by this group
     const int lg = warp & 3;
     const int row = lg * 32 + lane;            // query row in the tile == TMEM lane
-    const int gt = threadIdx.x - 64;           // 0..127 inside the group
+    const int gt = threadIdx.x - 64 - 128 * t; // 0..127 inside the group
+    float* mkg = mk + 2 * t * 2 * kAT;         // this group's staging: [buf][bias 128 | m 128]
+    uint64_t* sfull = s_full + 2 * t;
+    uint64_t* sempty = s_empty + 2 * t;
+    uint64_t* mkbar = mk_bar + 2 * t;
     int blk = 0;
-    int it = 0;
-    for (int item = blockIdx.x; item < p.n_items; item += gridDim.x, ++it) {
-      int b, h, qt;
-      decode_item(p, item, b, h, qt);
+    int ng = 0;                                // items this group has processed
+    for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+      const Item w = decode_item(p, item);
+      if (t >= w.nq) continue;
+      const int qt = w.qt0 + t;
       const int q = qt * kAT + row;             // query position in the sequence
       const int nkb = kblocks_of(p, qt);
-      float mrun = -CUDART_INF_F, l = 0.f, a = 0.f;
+      float mrun = -CUDART_INF_F;
+      float l4[4] = {0.f, 0.f, 0.f, 0.f}, a4[4] = {0.f, 0.f, 0.f, 0.f};
       bool ok = true;
+      // keys' (bias * log2 e, carried score) of block kb for thread gt, masked keys get -inf;
+      // loaded one block ahead so that the global round trip overlaps the current block
+      auto key_vals = [&](int kb, float& bias, float& m) {
+        const int key = kb * kAT + gt;
+        bias = -CUDART_INF_F;
+        m = 0.f;
+        if (key < p.S) {
+          const size_t tk = static_cast<size_t>(w.b) * p.S + key;
+          bias = p.key_bias ? __ldg(p.key_bias + tk) * 1.4426950408889634f : 0.f;
+          m = kFloatM ? __ldg(p.m_prev + tk) : static_cast<float>(__ldg(p.is_vision + tk) != 0);
+        }
+      };
+      float nb_bias, nb_m;
+      key_vals(0, nb_bias, nb_m);
       for (int kb = 0; kb < nkb; ++kb, ++blk) {
         const int buf = blk & 1;
         const uint32_t use = static_cast<uint32_t>(blk >> 1);
-        // stage this block's keys: (bias * log2 e, carried score), masked keys get -inf
-        {
-          const int key = kb * kAT + gt;
-          float bias = -CUDART_INF_F, m = 0.f;
-          if (key < p.S) {
-            const size_t t = static_cast<size_t>(b) * p.S + key;
-            bias = p.key_bias ? __ldg(p.key_bias + t) * 1.4426950408889634f : 0.f;
-            m = kFloatM ? __ldg(p.m_prev + t) : static_cast<float>(__ldg(p.is_vision + t) != 0);
-          }
-          mk[buf * kAT + gt] = make_float2(bias, m);
-          mbar_arrive(mk_bar + buf);
-        }
-        if (!mbar_wait(mk_bar + buf, use & 1u, wc)) { ok = false; break; }
-        if (!mbar_wait(s_full + buf, use & 1u, wc)) { ok = false; break; }
+        mkg[buf * 2 * kAT + gt] = nb_bias;
+        mkg[buf * 2 * kAT + kAT + gt] = nb_m;
+        mbar_arrive(mkbar + buf);
+        if (kb + 1 < nkb) key_vals(kb + 1, nb_bias, nb_m);
+        if (!mbar_wait(mkbar + buf, use & 1u, wc)) { ok = false; break; }
+        if (!mbar_wait(sfull + buf, use & 1u, wc)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t ta = tmem + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(buf * kAT);
-        const float2* mkb = mk + buf * kAT;
+        const uint32_t ta = tmem + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>((2 * t + buf) * kAT);
+        const float4* bias4 = reinterpret_cast<const float4*>(mkg + buf * 2 * kAT);
+        const float4* m4 = reinterpret_cast<const float4*>(mkg + buf * 2 * kAT + kAT);
         const bool diag = p.causal && kb == qt;
 #pragma unroll 1
         for (int c = 0; c < kAT / 32; ++c) {
           float v[32];
           tmem_ld32(ta + 32u * c, v);
-          float cmax = -CUDART_INF_F;
+          float cm[4] = {-CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F};
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int kc = c * 32 + i;
-            const float2 bm = mkb[kc];
-            float s = fmaf(v[i], p.scale_log2, bm.x);
-            if (diag && kc > row) s = -CUDART_INF_F;
-            v[i] = s;
-            cmax = fmaxf(cmax, s);
+          for (int i4 = 0; i4 < 8; ++i4) {
+            const float4 bb = bias4[c * 8 + i4];
+            const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
+            const int i = 4 * i4;
+            fma2(v[i], v[i + 1], v[i], v[i + 1], p.scale_log2, p.scale_log2, bv[0], bv[1]);
+            fma2(v[i + 2], v[i + 3], v[i + 2], v[i + 3], p.scale_log2, p.scale_log2, bv[2], bv[3]);
           }
-          const float mnew = fmaxf(mrun, cmax);
-          if (mnew != -CUDART_INF_F) {
-            const float corr = exp2f(mrun - mnew);
-            l *= corr;
-            a *= corr;
-            mrun = mnew;
+          if (diag) {                           // causal mask inside the diagonal block only
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float e = exp2f(v[i] - mnew);
-              l += e;
-              a = fmaf(e, mkb[c * 32 + i].y, a);
+            for (int i = 0; i < 32; ++i)
+              if (c * 32 + i > row) v[i] = -CUDART_INF_F;
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i) cm[i & 3] = fmaxf(cm[i & 3], v[i]);
+          const float mnew = fmaxf(mrun, fmaxf(fmaxf(cm[0], cm[1]), fmaxf(cm[2], cm[3])));
+          if (mnew != -CUDART_INF_F) {
+            if (mnew != mrun) {                 // rescale the running sums to the new maximum
+              const float corr = ex2(mrun - mnew);
+#pragma unroll
+              for (int u = 0; u < 4; ++u) {
+                l4[u] *= corr;
+                a4[u] *= corr;
+              }
+              mrun = mnew;
+            }
+#pragma unroll
+            for (int i4 = 0; i4 < 8; ++i4) {
+              const float4 mm = m4[c * 8 + i4];
+              const float mv[4] = {mm.x, mm.y, mm.z, mm.w};
+              const int i = 4 * i4;
+              float t0, t1, t2, t3;
+              add2(t0, t1, v[i], v[i + 1], -mnew, -mnew);
+              add2(t2, t3, v[i + 2], v[i + 3], -mnew, -mnew);
+              const float e0 = ex2(t0), e1 = ex2(t1), e2 = ex2(t2), e3 = ex2(t3);
+              add2(l4[0], l4[1], l4[0], l4[1], e0, e1);
+              add2(l4[2], l4[3], l4[2], l4[3], e2, e3);
+              fma2(a4[0], a4[1], e0, e1, mv[0], mv[1], a4[0], a4[1]);
+              fma2(a4[2], a4[3], e2, e3, mv[2], mv[3], a4[2], a4[3]);
             }
           }
         }
         tc_fence_before();
-        mbar_arrive(s_empty + buf);
+        mbar_arrive(sempty + buf);
       }
       if (!ok) break;
+      const float l = (l4[0] + l4[1]) + (l4[2] + l4[3]);
+      const float a = (a4[0] + a4[1]) + (a4[2] + a4[3]);
       // head result, then the head average of the tile by the last head to finish
       const bool valid = q < p.S;
-      const size_t tok = static_cast<size_t>(b) * p.S + q;
-      if (valid) p.part[static_cast<size_t>(h) * p.T + tok] = a / l;
+      const size_t tok = static_cast<size_t>(w.b) * p.S + q;
+      if (valid) p.part[static_cast<size_t>(w.h) * p.T + tok] = a / l;
       __threadfence();
-      mbar_arrive(out_bar);
+      const uint32_t nt = static_cast<uint32_t>(ng++);   // this item's phase of the group's barriers
+      mbar_arrive(out_bar + t);
       if (gt == 0) {
         uint32_t last = 0u;
-        if (mbar_wait(out_bar, static_cast<uint32_t>(it) & 1u, wc)) {
-          const uint32_t n = atomicAdd(p.ticket + b * p.n_qtiles + qt, 1u) + 1u;
+        if (mbar_wait(out_bar + t, nt & 1u, wc)) {
+          const uint32_t n = atomicAdd(p.ticket + w.b * p.n_qtiles + qt, 1u) + 1u;
           last = (n == static_cast<uint32_t>(p.H)) ? 1u : 0u;
-          if (last) p.ticket[b * p.n_qtiles + qt] = 0u;     // ready for the next call
+          if (last) p.ticket[w.b * p.n_qtiles + qt] = 0u;     // ready for the next call
         }
-        *decision = last;
-        mbar_arrive(dec_bar);
+        decision[t] = last;
+        mbar_arrive(dec_bar + t);
       }
-      if (!mbar_wait(dec_bar, static_cast<uint32_t>(it) & 1u, wc)) break;
-      if (*decision && valid) {
+      if (!mbar_wait(dec_bar + t, nt & 1u, wc)) break;
+      if (decision[t] && valid) {
         __threadfence();
         float sum = 0.f;
         for (int hh = 0; hh < p.H; ++hh) sum += __ldcg(p.part + static_cast<size_t>(hh) * p.T + tok);
@@ -286,7 +378,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem, 256);
+  if (warp == 1) tmem_dealloc(tmem, 512);
 }
 
 }  // namespace
@@ -296,11 +388,13 @@ cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const 
   if (p.hd != kHd) return cudaErrorNotSupported;
   const int n_ks = 4;
   const uint32_t smem = attn_layout(n_ks).total;
-  const int grid = p.n_items < n_sms ? p.n_items : n_sms;
+  if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
+  const int n_items = ((p.n_qtiles + 1) / 2) * p.B * p.H;
+  const int grid = n_items < n_sms ? n_items : n_sms;
   auto k = p.m_prev ? k_attn_mass<true> : k_attn_mass<false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k<<<grid, 192, smem, s>>>(tmQ, tmK, p, n_ks);
+  k<<<grid, 320, smem, s>>>(tmQ, tmK, p, n_ks);
   return cudaGetLastError();
 }
 
