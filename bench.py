@@ -7,9 +7,11 @@ A step is one pass of the whole router hot path over one batch of the workload:
 Default workload: the DeepSeekMoE-style VLM layer, T = 16384 tokens (8 x [576 image + 1472 text]),
 d = 2048, E = 64 routed experts, top-6, 8 bins, bf16. Inputs are seeded synthetic data.
 
-Timing: W warm-up steps, then K timed steps. Each call is replayed from a CUDA graph; before
-every step the L2 is flushed by writing a 256 MiB buffer (outside the timed interval), and CUDA
-events on the launching stream bracket each call. --gpus N under torchrun runs N independent
+Timing: W warm-up steps, then K timed steps. The step (all calls) is replayed from one CUDA
+graph; before every step the L2 is flushed by writing a 256 MiB buffer (outside the timed
+interval), and CUDA events on the launching stream bracket each step. A second pass of K steps
+replays a copy of the graph with an event after every call, for the per-call breakdown and the
+backward call's duration. --gpus N under torchrun runs N independent
 replicas (the path needs no collective); time = max over ranks.
 """
 from __future__ import annotations
@@ -294,21 +296,38 @@ def main():
 
     parts = ([("attn", score)] if use_attn else []) + [("fwd", fwd), ("bwd", bwd), ("permute", perm)]
 
-    # eager warm-up (also checks the device status once), then graph capture per call
+    # eager warm-up (also checks the device status once), then one CUDA graph for the whole step
+    # (the timed object) and a second copy with an event after every call (the per-call breakdown;
+    # event nodes between the calls stop the graph from overlapping their launches, so that copy
+    # runs a little slower and is timed in a pass of its own)
     for _ in range(2):
         for _, fn in parts:
             fn()
     code, _ = r.device_status()
     assert code == 0, f"device status {code}"
-    graphs = []
     s = torch.cuda.Stream(device=dev)
     s.wait_stream(torch.cuda.current_stream())
+    g_step = torch.cuda.CUDAGraph()
+    g_parts, part_graphs = None, []
     with torch.cuda.stream(s):
-        for _, fn in parts:
-            g = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(g, stream=s):
+        with torch.cuda.graph(g_step, stream=s):
+            for _, fn in parts:
                 fn()
-            graphs.append(g)
+        try:
+            ev_in = [torch.cuda.Event(enable_timing=True, external=True) for _ in range(len(parts) + 1)]
+            g_parts = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g_parts, stream=s):
+                ev_in[0].record()
+                for i, (_, fn) in enumerate(parts):
+                    fn()
+                    ev_in[i + 1].record()
+        except Exception:          # no event nodes in graphs: one graph per call instead
+            g_parts = None
+            for _, fn in parts:
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=s):
+                    fn()
+                part_graphs.append(g)
     torch.cuda.current_stream().wait_stream(s)
     torch.cuda.synchronize()
     # our kernels per step: attention 1, fwd 1 (+1 Gaussian coefficients on the fp32 path),
@@ -318,12 +337,25 @@ def main():
                          + (2 if f32 else 3) + 1)
 
     def step_timed():
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        g_step.replay()
+        b.record()
+        return a, b
+
+    def parts_timed():
+        """Durations (ms) of the step's calls, one step."""
+        if g_parts is not None:
+            g_parts.replay()
+            torch.cuda.synchronize()
+            return [ev_in[i].elapsed_time(ev_in[i + 1]) for i in range(len(parts))]
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(parts) + 1)]
         ev[0].record()
-        for i, g in enumerate(graphs):
+        for i, g in enumerate(part_graphs):
             g.replay()
             ev[i + 1].record()
-        return ev
+        torch.cuda.synchronize()
+        return [ev[i].elapsed_time(ev[i + 1]) for i in range(len(parts))]
 
     for _ in range(args.warmup):
         flush.zero_()
@@ -353,8 +385,17 @@ def main():
         dist.barrier()
     torch.cuda.synchronize()
     clk = clocks.stop() if not args.profile else {"sm_mhz": None, "note": "profile run"}
-    t_step = [e[0].elapsed_time(e[-1]) for e in evs]
-    t_part = {name: [e[i].elapsed_time(e[i + 1]) for e in evs] for i, (name, _) in enumerate(parts)}
+    t_step = [a.elapsed_time(b) for a, b in evs]
+    # per-call breakdown: the same steps again, each call bracketed by events
+    t_part = {name: [] for name, _ in parts}
+    for _ in range(args.steps):
+        flush.zero_()
+        for (name, _), t in zip(parts, parts_timed()):
+            t_part[name].append(t)
+    total_ms = max_over_ranks(float(np.sum(t_step)), world, dev)
+    ms_per_step = total_ms / args.steps
+    value = job_rate(wl.T, world, ms_per_step)
+
     t_bwd = t_part["bwd"]
     total_ms = max_over_ranks(float(np.sum(t_step)), world, dev)
     ms_per_step = total_ms / args.steps
@@ -431,6 +472,8 @@ def main():
                                   else "Gaussian score; ")
                                + "fwd + bwd (dW, dX) + bin permutation",
                    "l2": "flushed before every step (256 MiB write, outside the timed interval)",
+                   "timing": "one CUDA graph per step, events around each replay; breakdown_us and "
+                             "the backward duration from a second pass with events between calls",
                    "clocks": "nvidia-smi every 100 ms over a load window of ~0.5 s of steps "
                              "ending with the timed steps",
                    "parallelism": f"replicas x{world}"},

@@ -148,6 +148,8 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();                                 // Q, K and the outputs may be in use before this
+  pdl_trigger();
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
@@ -394,8 +396,7 @@ cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const 
   auto k = p.m_prev ? k_attn_mass<true> : k_attn_mass<false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k<<<grid, 320, smem, s>>>(tmQ, tmK, p, n_ks);
-  return cudaGetLastError();
+  return launch_pdl(k, dim3(grid), dim3(320), smem, s, tmQ, tmK, p, n_ks);
 }
 
 }  // namespace smoes

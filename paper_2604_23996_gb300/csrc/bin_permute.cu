@@ -69,6 +69,9 @@ __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
   __shared__ int disp[kMaxBins * kMaxBins];
   __shared__ int ecnt[2 * kMaxExperts];
   __shared__ int ok_s;
+  // launched without programmatic serialization (a cooperative grid): everything before it has
+  // completed, so the next kernel may be scheduled now
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = p.K;
   for (int e = threadIdx.x; e < p.E; e += kPermThreads) {

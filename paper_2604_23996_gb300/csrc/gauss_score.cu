@@ -20,8 +20,9 @@ namespace {
 __global__ void __launch_bounds__(256) k_gauss_coef(const float* __restrict__ mu,
                                                     const float* __restrict__ var, int d, int dcoef,
                                                     float* __restrict__ coef, uint32_t* status) {
-  pdl_trigger();                            // the consumer may start its own prologue now
   __shared__ float red[8];
+  pdl_wait();
+  pdl_trigger();                            // the consumer may start its own prologue now
   const int i = blockIdx.x * 256 + threadIdx.x;
   float a = 0.f, b = 0.f, c = 0.f;
   if (i < d && !gauss_coef_feature(mu[i], mu[d + i], var[i], var[d + i], a, b, c))
@@ -45,6 +46,7 @@ __global__ void __launch_bounds__(256) k_gauss_score(const GaussParams p) {
   float* ga = gsm;
   float* gb = ga + dpad;
   pdl_wait();                               // coefficients of the kernel launched just before
+  pdl_trigger();
   for (int i = threadIdx.x; i < dpad; i += 256) {
     ga[i] = p.gcoef[i];
     gb[i] = p.gcoef[p.dcoef + i];
@@ -110,8 +112,7 @@ __global__ void __launch_bounds__(256) k_gauss_score(const GaussParams p) {
 
 cudaError_t launch_gauss_coef(const float* mu, const float* var, int d, int dcoef, float* coef,
                               uint32_t* status, cudaStream_t s) {
-  k_gauss_coef<<<dcoef / 256, 256, 0, s>>>(mu, var, d, dcoef, coef, status);
-  return cudaGetLastError();
+  return launch_pdl(k_gauss_coef, dim3(dcoef / 256), dim3(256), 0, s, mu, var, d, dcoef, coef, status);
 }
 
 cudaError_t launch_gauss_score(const GaussParams& p, smoes_dtype dt, int n_sms, cudaStream_t s) {
@@ -123,17 +124,7 @@ cudaError_t launch_gauss_score(const GaussParams& p, smoes_dtype dt, int n_sms, 
   auto k = (dt == SMOES_BF16) ? k_gauss_score<true> : k_gauss_score<false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
-  cfg.blockDim = dim3(256);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k, p);
+  return launch_pdl(k, dim3(grid), dim3(256), smem, s, p);
 }
 
 }  // namespace smoes

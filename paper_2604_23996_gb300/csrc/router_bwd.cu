@@ -91,6 +91,8 @@ __device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
 // experts lie in at most two bins: their coefficients are read once per bin.
 template <int TPT>
 __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
+  pdl_wait();                                         // scores and tables of the forward
+  pdl_trigger();
   const Dims& dm = p.dm;
   const int E = dm.E, K = dm.K, k = dm.k;
   constexpr int kEp = TPT * 8;
@@ -260,14 +262,19 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   const uint32_t tm_dx = tmem + 256u;          // two 64-column dX^T buffers after the dW^T blocks
+  if (warp == 0 && lane == 0) {
+    // W slice (atom a = columns d0 + 64a .. +64), requested before the dz prep kernel has
+    // finished: that kernel does not write W, and it started only after all earlier work
+    mbar_arrive_expect_tx(wfull, static_cast<uint32_t>(nb) * 2u * dz_half);
+    for (int a = 0; a < 2 * nb; ++a) tma_load_2d(wsl + a * dz_half, &tmW, wfull, d0 + 64 * a, 0);
+  }
+  pdl_wait();                                  // the dz images, X and dX
+  pdl_trigger();
 
   if (warp == 0) {
     // -------------------------------------------------------------- TMA producer
     if (lane == 0) {
       bool ok = true;
-      mbar_arrive_expect_tx(wfull, static_cast<uint32_t>(nb) * 2u * dz_half);
-      for (int a = 0; a < 2 * nb; ++a)        // W slice: atom a = columns d0 + 64a .. +64
-        tma_load_2d(wsl + a * dz_half, &tmW, wfull, d0 + 64 * a, 0);
       int st = 0;
       uint32_t ph = 0;
       long issued = 0, dz_issued = 0;
@@ -442,6 +449,8 @@ constexpr int kF32MaxE = 64;
 __global__ void __launch_bounds__(256)
 k_router_bwd_f32(const BwdParams p) {
   extern __shared__ float bs[];
+  pdl_wait();
+  pdl_trigger();
   const Dims& dm = p.dm;
   const int E = dm.E, K = dm.K, k = dm.k;
   float* dzs = bs;                                   // [64][E+1]
@@ -527,6 +536,8 @@ constexpr int kDwCols = 32;
 
 __global__ void __launch_bounds__(kDwSlices * kDwCols) k_dw_reduce(const BwdParams p) {
   __shared__ float4 part_s[kDwSlices][kDwCols];
+  pdl_wait();                                              // the partials of the main kernel
+  pdl_trigger();
   const size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
   const bool vec = (n & 3) == 0;
   const size_t nv = vec ? n / 4 : n;                       // float4 (or scalar) columns
@@ -584,10 +595,9 @@ cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s) {
   const int E_pad = round_up(p.dm.E, 64);
   const long threads = static_cast<long>(p.n_tiles) * kBwdBT * (E_pad / 8);
   const int blocks = static_cast<int>((threads + 255) / 256);
-  if (E_pad == 64) k_dz_prep<8><<<blocks, 256, 0, s>>>(p);
-  else if (E_pad == 128) k_dz_prep<16><<<blocks, 256, 0, s>>>(p);
-  else return cudaErrorInvalidValue;
-  return cudaGetLastError();
+  if (E_pad == 64) return launch_pdl(k_dz_prep<8>, dim3(blocks), dim3(256), 0, s, p);
+  if (E_pad == 128) return launch_pdl(k_dz_prep<16>, dim3(blocks), dim3(256), 0, s, p);
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, const CUtensorMap& tmW,
@@ -601,24 +611,21 @@ cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, c
   auto k = (E_pad == 64) ? k_router_bwd_tc<64> : k_router_bwd_tc<128>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k<<<p.groups * p.slices, 192, smem, s>>>(tmX, tmW, tmDX, p, n_xst);
-  return cudaGetLastError();
+  return launch_pdl(k, dim3(p.groups * p.slices), dim3(192), smem, s, tmX, tmW, tmDX, p, n_xst);
 }
 
 
 cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s) {
   if (p.dm.E > kF32MaxE) return cudaErrorInvalidValue;
   const size_t smem = sizeof(float) * 64 * (p.dm.E + 1);
-  k_router_bwd_f32<<<p.n_tiles, 256, smem, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(k_router_bwd_f32, dim3(p.n_tiles), dim3(256), smem, s, p);
 }
 
 cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s) {
   size_t n = static_cast<size_t>(p.dm.E) * p.dm.d;
   if ((n & 3) == 0) n /= 4;
   const int blocks = static_cast<int>((n + kDwCols - 1) / kDwCols);
-  k_dw_reduce<<<blocks, kDwSlices * kDwCols, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(k_dw_reduce, dim3(blocks), dim3(kDwSlices * kDwCols), 0, s, p);
 }
 
 }  // namespace smoes

@@ -614,6 +614,9 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // X, W, the statistics and the outputs may be in use by the kernel before this one
+  pdl_wait();
+  pdl_trigger();
 
   if (kGauss && warp >= 2) {
     // this CTA's Gaussian coefficients (eqs. 8-9), computed by the epilogue and Gaussian warps
@@ -851,6 +854,8 @@ k_router_fwd_f32(const FwdParams p) {
   const int t = threadIdx.x, r = t >> 2, qd = t & 3;
   const int tile = blockIdx.x;
   const int j0 = tile * kTileRows;
+  pdl_wait();
+  pdl_trigger();
   if (t == 0) {
     *abort_flag = 0;
     mbar_init(bars + 0, 128);
@@ -958,8 +963,8 @@ cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
     auto k = gauss ? k_router_fwd_tc<true, KM> : k_router_fwd_tc<false, KM>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k<<<grid, gauss ? 320 : 192, smem, s>>>(tmX, tmW, tg, p, N, n_stages, use_stg ? 1 : 0);
-    return cudaGetLastError();
+    return launch_pdl(k, dim3(grid), dim3(gauss ? 320 : 192), smem, s, tmX, tmW, tg, p, N, n_stages,
+                      use_stg ? 1 : 0);
   });
 }
 
@@ -973,8 +978,7 @@ cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s) {
     auto k = gauss ? k_router_fwd_f32<true, KM> : k_router_fwd_f32<false, KM>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k<<<p.n_tiles, 512, smem, s>>>(p);
-    return cudaGetLastError();
+    return launch_pdl(k, dim3(p.n_tiles), dim3(512), smem, s, p);
   });
 }
 

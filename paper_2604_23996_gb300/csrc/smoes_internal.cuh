@@ -163,6 +163,29 @@ struct StaticPermScratch {
 cudaError_t static_perm_scratch(StaticPermScratch** out);
 
 // ------------------------------------------------------------------ launchers (in .cu files)
+// Every kernel of the library is launched with programmatic stream serialization: its CTAs may
+// be scheduled while the kernel before it in the stream is finishing, which hides the launch
+// latency between the calls of a step. The protocol that keeps this exact: a kernel calls
+// pdl_wait() before it reads or writes memory that any earlier work in the stream may touch,
+// and pdl_trigger() only after its own pdl_wait(), so that a kernel that starts early knows
+// that every kernel before its immediate predecessor has completed; only data that the
+// immediate predecessor does not write (a plan table, W in the backward) is read earlier.
+template <class... KArgs, class... Args>
+cudaError_t launch_pdl(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k, static_cast<Args&&>(args)...);
+}
+
 // tmG: TMA map of the saved softmax scores [T, E] fp32 (box 32 x 128, 128-byte swizzle), or
 // null to store them row by row.
 cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
