@@ -2,8 +2,9 @@
 """Router fwd+bwd throughput of the SMoES hot path on GB300 (one JSON line on stdout).
 
 A step is one pass of the whole router hot path over one batch of the workload:
-  smoes_router_fwd (gate GEMM + Gaussian modality score + softmax/top-k/bins + per-sample MI)
-  -> smoes_router_bwd (MI gradient -> dW and dX) -> smoes_bin_permute (de-duplicated dispatch).
+  smoes_router_fwd_permute (gate GEMM + Gaussian modality score + softmax/top-k/bins + per-sample
+  MI + the de-duplicated bin dispatch of the top-k, one launch) -> smoes_router_bwd (MI gradient
+  -> dW and dX).
 Default workload: the DeepSeekMoE-style VLM layer, T = 16384 tokens (8 x [576 image + 1472 text]),
 d = 2048, E = 64 routed experts, top-6, 8 bins, bf16. Inputs are seeded synthetic data.
 
@@ -282,19 +283,17 @@ def main():
     def score():
         r.modality_score(bd.SMOES_SCORE_ATTN, Ma, attn=attn)
 
-    def fwd():
+    def fwd_perm():
+        # the forward and the bin permutation of its top-k: one launch on the bf16 path
         if use_attn:
-            r.forward(X, W, M_in=Ma, bin_prob=False)
+            r.forward_permute(X, W, M_in=Ma, bin_prob=False, is_vision=is_vis)
         else:
-            r.forward(X, W, mu=mu, var=var, tau=wl.tau, bin_prob=False)
+            r.forward_permute(X, W, mu=mu, var=var, tau=wl.tau, bin_prob=False, is_vision=is_vis)
 
     def bwd():
         r.backward(X, W, Ma if use_attn else r.M, dW, dX=dX, loss_scale=1e-4)
 
-    def perm():
-        r.permute(is_vision=is_vis)
-
-    parts = ([("attn", score)] if use_attn else []) + [("fwd", fwd), ("bwd", bwd), ("permute", perm)]
+    parts = ([("attn", score)] if use_attn else []) + [("fwd+permute", fwd_perm), ("bwd", bwd)]
 
     # eager warm-up (also checks the device status once), then one CUDA graph for the whole step
     # (the timed object) and a second copy with an event after every call (the per-call breakdown;
@@ -330,11 +329,11 @@ def main():
                 part_graphs.append(g)
     torch.cuda.current_stream().wait_stream(s)
     torch.cuda.synchronize()
-    # our kernels per step: attention 1, fwd 1 (+1 Gaussian coefficients on the fp32 path),
-    # bwd 3 (dz prep, main, dW reduce; fp32: main, dW reduce), permutation 1
+    # our kernels per step: attention 1; fwd + permutation 2 (forward, scatter; fp32: Gaussian
+    # coefficients 1, forward 1, permutation 1); bwd 3 (dz prep, main, dW reduce; fp32: main, dW reduce)
     f32 = dtype != bd.SMOES_BF16
-    launches_per_step = ((1 if use_attn else 0) + 1 + (1 if f32 and not use_attn else 0)
-                         + (2 if f32 else 3) + 1)
+    fwd_launches = ((0 if use_attn else 1) + 2) if f32 else 2
+    launches_per_step = (1 if use_attn else 0) + fwd_launches + (2 if f32 else 3)
 
     def step_timed():
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)

@@ -157,6 +157,24 @@ smoes_status smoes_router_fwd(smoes_plan plan, const void* X, const void* W, con
                               float* joint, float* mi, float* loss,
                               void* ws, size_t ws_bytes, cudaStream_t stream);
 
+/* (2b) The forward (2) and the bin permutation (4) of its own top-k in one launch.
+ *   Arguments: those of smoes_router_fwd, then those of smoes_bin_permute (topk_idx is the
+ *   forward's output); results are identical to smoes_router_fwd followed by smoes_bin_permute.
+ *   On bf16 plans the forward kernel counts each CTA's (token, bin) pairs from the top-k it holds
+ *   in registers; after a grid-wide barrier (a cooperative launch: every CTA resident) the warps
+ *   that are idle once the CTA's gate GEMM is done place the CTA's entries, while the per-sample
+ *   MI reduction of eqs. (12)-(15) runs. fp32 plans make the two calls. The paper has no
+ *   counterpart for this fusion; it removes the separate launch and counting pass. */
+smoes_status smoes_router_fwd_permute(smoes_plan plan, const void* X, const void* W,
+                                      const float* M_in, const smoes_gauss_args* gauss,
+                                      float* M_out, int32_t* topk_idx, float* topk_w,
+                                      float* bin_prob, float* joint, float* mi, float* loss,
+                                      const int32_t* home, const uint8_t* is_vision,
+                                      int32_t* bin_offsets, int32_t* perm_token,
+                                      uint32_t* perm_mask, int32_t* dispatch,
+                                      int32_t* expert_counts, void* ws, size_t ws_bytes,
+                                      cudaStream_t stream);
+
 /* (3) Backward of loss_scale * L_MI (plus, optionally, an upstream gradient of topk_w).
  *   The soft scores are constants (no gradient flows into M). X, W, M and topk_idx must be the
  *   tensors of the preceding smoes_router_fwd on the same ws.

@@ -67,6 +67,9 @@ _sig = {
     "smoes_modality_score": (_i, [_vp, _i, C.POINTER(ScoreArgs), _vp, _vp, _sz, _vp]),
     "smoes_router_fwd": (_i, [_vp, _vp, _vp, _vp, C.POINTER(GaussArgs), _vp, _vp, _vp, _vp, _vp,
                               _vp, _vp, _vp, _sz, _vp]),
+    "smoes_router_fwd_permute": (_i, [_vp, _vp, _vp, _vp, C.POINTER(GaussArgs), _vp, _vp, _vp, _vp,
+                                      _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz,
+                                      _vp]),
     "smoes_router_bwd": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _f, _vp, _i, _vp, _vp, _vp, _sz, _vp]),
     "smoes_bin_permute": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "smoes_bin_permute_noalloc": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -159,6 +162,22 @@ def smoes_router_fwd(plan, X, W, M_in, gauss, M_out, topk_idx, topk_w, bin_prob,
                                  _stream(stream))
 
 
+def smoes_router_fwd_permute(plan, X, W, M_in, gauss, M_out, topk_idx, topk_w, bin_prob, joint, mi,
+                             loss, home, is_vision, bin_offsets, perm_token, perm_mask, dispatch,
+                             expert_counts, ws, stream=None) -> int:
+    """smoes_router_fwd and smoes_bin_permute of its top-k in one call (one launch on bf16)."""
+    g = None
+    if gauss is not None:
+        g = GaussArgs(None, _p(gauss["mu"]), _p(gauss["var"]), float(gauss.get("tau", 0.0)))
+    return _lib.smoes_router_fwd_permute(plan, _p(X), _p(W), _p(M_in),
+                                         None if g is None else C.byref(g), _p(M_out),
+                                         _p(topk_idx), _p(topk_w), _p(bin_prob), _p(joint),
+                                         _p(mi), _p(loss), _p(home), _p(is_vision),
+                                         _p(bin_offsets), _p(perm_token), _p(perm_mask),
+                                         _p(dispatch), _p(expert_counts), _p(ws),
+                                         ws.numel() * ws.element_size(), _stream(stream))
+
+
 def smoes_router_bwd(plan, X, W, M, topk_idx, d_topk_w, loss_scale, dW, accumulate_dW, dX,
                      dlogits, ws, stream=None) -> int:
     return _lib.smoes_router_bwd(plan, _p(X), _p(W), _p(M), _p(topk_idx), _p(d_topk_w),
@@ -230,6 +249,17 @@ class Router:
                                 self.topk_idx, self.topk_w, self.bin_prob if bin_prob else None,
                                 self.joint, self.mi, self.loss, self.ws, stream)
         _check(code, "smoes_router_fwd")
+
+    def forward_permute(self, X, W, M_in=None, mu=None, var=None, tau=0.0, bin_prob=True,
+                        is_vision=None, home=None, stream=None):
+        """forward() then permute() of its top-k, fused into one launch on bf16 plans."""
+        gauss = None if M_in is not None else dict(mu=mu, var=var, tau=tau)
+        code = smoes_router_fwd_permute(
+            self.plan, X, W, M_in, gauss, None if M_in is not None else self.M, self.topk_idx,
+            self.topk_w, self.bin_prob if bin_prob else None, self.joint, self.mi, self.loss, home,
+            is_vision, self.bin_offsets, self.perm_token, self.perm_mask, self.dispatch,
+            self.expert_counts if is_vision is not None else None, self.ws, stream)
+        _check(code, "smoes_router_fwd_permute")
 
     def backward(self, X, W, M, dW, dX=None, dlogits=None, loss_scale=1.0, d_topk_w=None,
                  accumulate=False, stream=None):

@@ -24,7 +24,7 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 struct Layout {
   size_t status, sample_ticket, loss_ticket, offsets, token_sample, expert_bin, expert_slot,
       piece_base, sample_pieces, pieces, mi32, tabs, gsave, dw_part, dz_img, perm, attn_ticket, attn_part,
-      gcoef, perm_sync;
+      gcoef, perm_sync, fperm;
   size_t header_bytes;   // [0, header_bytes) is cleared by smoes_workspace_init
   size_t total;
 };
@@ -160,6 +160,67 @@ smoes_status check_ws(const smoes_plan_s* P, const void* ws, size_t ws_bytes) {
 
 smoes_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SMOES_OK : SMOES_ERR_CUDA; }
 
+// The forward of smoes_router_fwd; perm: the fused permutation's outputs (tensor-core path), or null.
+smoes_status router_fwd(smoes_plan P, const void* X, const void* W, const float* M_in,
+                        const smoes_gauss_args* gauss, float* M_out, int32_t* topk_idx,
+                        float* topk_w, float* bin_prob, float* joint, float* mi, float* loss,
+                        const FusedPerm* perm, void* ws, size_t ws_bytes, cudaStream_t stream) {
+  if (!P) return SMOES_ERR_INVALID_ARG;
+  smoes_status st = check_ws(P, ws, ws_bytes);
+  if (st != SMOES_OK) return st;
+  const smoes_router_desc& d = P->desc;
+  if (!loss) return SMOES_ERR_INVALID_ARG;
+  if (d.T == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), stream));
+  if (!X || !W || !topk_idx || !topk_w || !mi) return SMOES_ERR_INVALID_ARG;
+  if ((M_in == nullptr) == (gauss == nullptr)) return SMOES_ERR_INVALID_ARG;
+  if (gauss && (!gauss->mu || !gauss->var || !M_out)) return SMOES_ERR_INVALID_ARG;
+  if (!aligned16(X) || !aligned16(W) || (M_in && !aligned16(M_in)) || (M_out && !aligned16(M_out)) ||
+      (gauss && (!aligned16(gauss->mu) || !aligned16(gauss->var))))
+    return SMOES_ERR_ALIGNMENT;
+  if (d.dtype == SMOES_F32 && d.E > 64) return SMOES_ERR_UNSUPPORTED;
+
+  FwdParams p{};
+  p.dm = make_dims(P);
+  p.ws = make_view(P, ws);
+  p.X = X;
+  p.W = W;
+  p.M_in = M_in;
+  p.mu = gauss ? gauss->mu : nullptr;
+  p.var = gauss ? gauss->var : nullptr;
+  p.inv_tau = gauss ? 1.f / (gauss->tau > 0.f ? gauss->tau : 0.5f * d.d) : 1.f;
+  p.M_out = gauss ? M_out : nullptr;
+  p.topk_idx = topk_idx;
+  p.topk_w = topk_w;
+  p.bin_prob = bin_prob;
+  p.joint = joint;
+  p.mi = mi;
+  p.loss = loss;
+  p.limit_ns = kWaitLimitNs;
+  if (perm) {
+    p.perm = *perm;
+    p.perm.cta_counts = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + P->L.fperm);
+    p.perm.sync = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + P->L.perm_sync);
+  }
+  if (gauss && d.dtype == SMOES_F32) {
+    const cudaError_t e = launch_gauss_coef(gauss->mu, gauss->var, d.d, p.ws.dcoef, p.ws.gcoef,
+                                            p.ws.status, stream);
+    if (e != cudaSuccess) return SMOES_ERR_CUDA;
+  }
+  if (d.dtype == SMOES_BF16) {
+    p.n_tiles = (d.T + kFwdBM - 1) / kFwdBM;
+    CUtensorMap tx, tw;
+    if (!encode_bf16_2d(&tx, X, d.T, d.d, kFwdBM, kFwdBK, true) ||
+        !encode_bf16_2d(&tw, W, d.E, d.d, round_up(d.E, 16), kFwdBK, true))
+      return SMOES_ERR_CUDA;
+    // saved scores leave through TMA when their rows are 16-byte multiples
+    CUtensorMap tg;
+    const bool tma_g = d.E % 4 == 0 && d.E <= 128 && encode_f32_2d(&tg, p.ws.gsave, d.T, d.E, 128, 32, true);
+    return cuda_status(launch_router_fwd_bf16(p, tx, tw, tma_g ? &tg : nullptr, P->n_sms, stream));
+  }
+  p.n_tiles = P->n_groups;
+  return cuda_status(launch_router_fwd_f32(p, stream));
+}
+
 }  // namespace
 
 extern "C" {
@@ -287,6 +348,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.dz_img = take(d.dtype == SMOES_BF16 && E <= 128
                       ? static_cast<size_t>(P->bwd_tiles) * 2 * round_up(E, 64) * 128 : 0);
   L.perm = take(sizeof(int32_t) * static_cast<size_t>(P->perm_nblocks) * K);
+  L.fperm = take(sizeof(int32_t) * static_cast<size_t>(std::max(P->n_sms, 1)) * K);   // per-CTA counts
   L.attn_part = take(sizeof(float) * static_cast<size_t>(T) * std::max(0, d.attn_max_heads));
   L.gcoef = take(sizeof(float) * (2 * static_cast<size_t>(P->dcoef) + P->dcoef / 256));
   L.total = o;
@@ -407,55 +469,41 @@ smoes_status smoes_router_fwd(smoes_plan P, const void* X, const void* W, const 
                               const smoes_gauss_args* gauss, float* M_out, int32_t* topk_idx,
                               float* topk_w, float* bin_prob, float* joint, float* mi, float* loss,
                               void* ws, size_t ws_bytes, cudaStream_t stream) {
-  if (!P) return SMOES_ERR_INVALID_ARG;
-  smoes_status st = check_ws(P, ws, ws_bytes);
-  if (st != SMOES_OK) return st;
-  const smoes_router_desc& d = P->desc;
-  if (!loss) return SMOES_ERR_INVALID_ARG;
-  if (d.T == 0) return cuda_status(cudaMemsetAsync(loss, 0, sizeof(float), stream));
-  if (!X || !W || !topk_idx || !topk_w || !mi) return SMOES_ERR_INVALID_ARG;
-  if ((M_in == nullptr) == (gauss == nullptr)) return SMOES_ERR_INVALID_ARG;
-  if (gauss && (!gauss->mu || !gauss->var || !M_out)) return SMOES_ERR_INVALID_ARG;
-  if (!aligned16(X) || !aligned16(W) || (M_in && !aligned16(M_in)) || (M_out && !aligned16(M_out)) ||
-      (gauss && (!aligned16(gauss->mu) || !aligned16(gauss->var))))
-    return SMOES_ERR_ALIGNMENT;
-  if (d.dtype == SMOES_F32 && d.E > 64) return SMOES_ERR_UNSUPPORTED;
+  return router_fwd(P, X, W, M_in, gauss, M_out, topk_idx, topk_w, bin_prob, joint, mi, loss,
+                    nullptr, ws, ws_bytes, stream);
+}
 
-  FwdParams p{};
-  p.dm = make_dims(P);
-  p.ws = make_view(P, ws);
-  p.X = X;
-  p.W = W;
-  p.M_in = M_in;
-  p.mu = gauss ? gauss->mu : nullptr;
-  p.var = gauss ? gauss->var : nullptr;
-  p.inv_tau = gauss ? 1.f / (gauss->tau > 0.f ? gauss->tau : 0.5f * d.d) : 1.f;
-  p.M_out = gauss ? M_out : nullptr;
-  p.topk_idx = topk_idx;
-  p.topk_w = topk_w;
-  p.bin_prob = bin_prob;
-  p.joint = joint;
-  p.mi = mi;
-  p.loss = loss;
-  p.limit_ns = kWaitLimitNs;
-  if (gauss && d.dtype == SMOES_F32) {
-    const cudaError_t e = launch_gauss_coef(gauss->mu, gauss->var, d.d, p.ws.dcoef, p.ws.gcoef,
-                                            p.ws.status, stream);
-    if (e != cudaSuccess) return SMOES_ERR_CUDA;
+smoes_status smoes_router_fwd_permute(smoes_plan P, const void* X, const void* W, const float* M_in,
+                                      const smoes_gauss_args* gauss, float* M_out,
+                                      int32_t* topk_idx, float* topk_w, float* bin_prob,
+                                      float* joint, float* mi, float* loss, const int32_t* home,
+                                      const uint8_t* is_vision, int32_t* bin_offsets,
+                                      int32_t* perm_token, uint32_t* perm_mask, int32_t* dispatch,
+                                      int32_t* expert_counts, void* ws, size_t ws_bytes,
+                                      cudaStream_t stream) {
+  if (!P) return SMOES_ERR_INVALID_ARG;
+  const smoes_router_desc& d = P->desc;
+  if (!bin_offsets || !dispatch) return SMOES_ERR_INVALID_ARG;
+  if (expert_counts && !is_vision) return SMOES_ERR_INVALID_ARG;
+  if (d.T > 0 && (!perm_token || !perm_mask)) return SMOES_ERR_INVALID_ARG;
+  // inside the forward launch on the tensor-core path; otherwise the two calls in order
+  if (d.dtype == SMOES_BF16 && d.T > 0 && d.n_bins <= kMaxBins && d.E <= kMaxExperts) {
+    FusedPerm f{};
+    f.home = home;
+    f.is_vision = is_vision;
+    f.bin_offsets = bin_offsets;
+    f.perm_token = perm_token;
+    f.perm_mask = perm_mask;
+    f.dispatch = dispatch;
+    f.expert_counts = expert_counts;
+    return router_fwd(P, X, W, M_in, gauss, M_out, topk_idx, topk_w, bin_prob, joint, mi, loss,
+                      &f, ws, ws_bytes, stream);
   }
-  if (d.dtype == SMOES_BF16) {
-    p.n_tiles = (d.T + kFwdBM - 1) / kFwdBM;
-    CUtensorMap tx, tw;
-    if (!encode_bf16_2d(&tx, X, d.T, d.d, kFwdBM, kFwdBK, true) ||
-        !encode_bf16_2d(&tw, W, d.E, d.d, round_up(d.E, 16), kFwdBK, true))
-      return SMOES_ERR_CUDA;
-    // saved scores leave through TMA when their rows are 16-byte multiples
-    CUtensorMap tg;
-    const bool tma_g = d.E % 4 == 0 && d.E <= 128 && encode_f32_2d(&tg, p.ws.gsave, d.T, d.E, 128, 32, true);
-    return cuda_status(launch_router_fwd_bf16(p, tx, tw, tma_g ? &tg : nullptr, P->n_sms, stream));
-  }
-  p.n_tiles = P->n_groups;
-  return cuda_status(launch_router_fwd_f32(p, stream));
+  smoes_status st = router_fwd(P, X, W, M_in, gauss, M_out, topk_idx, topk_w, bin_prob, joint, mi,
+                               loss, nullptr, ws, ws_bytes, stream);
+  if (st != SMOES_OK) return st;
+  return smoes_bin_permute(P, topk_idx, home, is_vision, bin_offsets, perm_token, perm_mask,
+                           dispatch, expert_counts, ws, ws_bytes, stream);
 }
 
 smoes_status smoes_router_bwd(smoes_plan P, const void* X, const void* W, const float* M,

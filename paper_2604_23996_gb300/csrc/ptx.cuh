@@ -101,6 +101,8 @@ __device__ inline bool grid_barrier(uint32_t* sync, uint32_t n, uint64_t limit_n
   }
   const uint64_t t0 = global_ns();
   while (*gen == g0) {
+    __nanosleep(128);         // one polling load per block every ~0.1 us: the word's L2 slice
+                              // also serves other traffic
     if (global_ns() - t0 > limit_ns) {
       atomicOr(status, 2u);   // the timeout status bit
       return false;
@@ -108,6 +110,11 @@ __device__ inline bool grid_barrier(uint32_t* sync, uint32_t n, uint64_t limit_n
   }
   __threadfence();
   return true;
+}
+
+// Named barrier `id` (1..15) over `n` threads of the CTA (n a multiple of 32).
+__device__ __forceinline__ void named_bar(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
 
 // ---------------------------------------------------------------------------------- TMA

@@ -29,6 +29,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr int kTileRows = kPieceTokens;      // 128 tokens per tile and per partial-sum piece
 constexpr int kPsStride = kTileRows + 1;     // padded row of the per-bin / per-modality tables
 constexpr int kMaxNV = piece_values(kMaxBins);
+constexpr int kCoefBars = 8;                 // Gaussian coefficient chunks with their own barrier
 
 // Top-k selection key: the logit with its low `ib` mantissa bits replaced by the expert index,
 // (2^ib - 1 - e) for a non-negative logit and e for a negative one, so that as floats the keys
@@ -263,8 +264,10 @@ struct EpiSmem {
   float* m_s;            // [5][kPsStride] (M_v - 1/2, M_t - 1/2, M_v, M_t, 1) of the tile's rows
   float* wpart;          // [2][4][kMaxNV] per-warp partial piece sums (double buffer)
   float* red;            // [kMaxNV] sample-reduce scratch of the group's first warp
+  int* ctot;             // [kMaxBins] (token, bin) pairs of the CTA's tiles (fused permutation)
   uint64_t* bar_in;      // count 128: the warps' partials of one (tile, sample) are written
   uint64_t* bar_out;     // count 128: the tile's pieces are written
+  uint64_t* perm_go;     // count 1: the CTA's top-k and pair counts are complete
   // optional staging of the tile's softmax scores for one coalesced TMA store: 32-column blocks
   // of [128 rows][128 bytes], 16-byte chunks swizzled by row (the 128-byte TMA swizzle)
   uint8_t* stg;          // null: scores are stored row by row
@@ -274,7 +277,7 @@ struct EpiSmem {
 };
 
 __host__ __device__ inline size_t epi_smem_floats(int K) {
-  return static_cast<size_t>(K) * kPsStride + 5u * kPsStride + 2u * 4u * kMaxNV + kMaxNV;
+  return static_cast<size_t>(K) * kPsStride + 5u * kPsStride + 2u * 4u * kMaxNV + kMaxNV + kMaxBins;
 }
 
 __device__ inline EpiSmem epi_smem(float* base, int K, uint64_t* bar_in, uint64_t* bar_out) {
@@ -283,8 +286,10 @@ __device__ inline EpiSmem epi_smem(float* base, int K, uint64_t* bar_in, uint64_
   es.m_s = es.p_s + K * kPsStride;
   es.wpart = es.m_s + 5 * kPsStride;
   es.red = es.wpart + 2 * 4 * kMaxNV;
+  es.ctot = reinterpret_cast<int*>(es.red + kMaxNV);
   es.bar_in = bar_in;
   es.bar_out = bar_out;
+  es.perm_go = nullptr;
   es.stg = nullptr;
   es.stg_full = es.stg_free = nullptr;
   es.tmG = nullptr;
@@ -296,11 +301,13 @@ __device__ inline EpiSmem epi_smem(float* base, int K, uint64_t* bar_in, uint64_
 // called after the last logit read. row: token row in
 // the tile (0..127, the thread's index in the group); lt: index of the tile among those this
 // group processes; meta: the tile's metadata (load_tile_meta); n_in: completed phases of
-// bar_in (identical in all 128 threads).
+// bar_in (identical in all 128 threads). With the fused permutation every warp adds its rows'
+// (token, bin) pairs to es.ctot, and after the CTA's last tile the first warp arrives on
+// es.perm_go once all rows are counted.
 template <int KM, class Src, class Release>
 __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release& release, int tile,
                               int row, int lt, float dll, const TileMeta& meta, const EpiSmem& es,
-                              const WaitCtx& wc, uint32_t& n_in) {
+                              const WaitCtx& wc, uint32_t& n_in, bool last_tile) {
   const Dims& dm = p.dm;
   const int E = dm.E, K = dm.K, k = dm.k;
   const int wg = row >> 5, lane = row & 31;
@@ -457,6 +464,22 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
   } else {
     for (int b = 0; b < K; ++b) prow[b * kPsStride] = 0.f;
   }
+  if (p.perm.perm_token) {           // (token, bin) pairs of this warp's rows, per bin
+    uint32_t bins = 0u;
+    if (valid) {
+#pragma unroll
+      for (int i = 0; i < KM; ++i) {
+        if (i < k) {
+          const int e = topk_index(tk[i], imask);
+          bins |= 1u << (dm.contig_bins ? e / dm.N_B : __ldg(p.ws.expert_bin + e));
+        }
+      }
+    }
+    for (int kb = 0; kb < K; ++kb) {
+      const int c = __popc(__ballot_sync(0xffffffffu, (bins >> kb) & 1u));
+      if (lane == kb && c) atomicAdd(es.ctot + kb, c);
+    }
+  }
   float* mrow = es.m_s + row;
   mrow[0] = dv;
   mrow[kPsStride] = dt;
@@ -505,6 +528,8 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
     if (lane == 0) ok = mbar_wait(es.bar_out, static_cast<uint32_t>(lt & 1), wc);
     ok = __shfl_sync(0xffffffffu, ok, 0);
     if (!ok) return;
+    // every row of the CTA's last tile is done: its top-k and pair counts may be read
+    if (p.perm.perm_token && last_tile && lane == 0) mbar_arrive(es.perm_go);
     for (int s = s0; s <= s1; ++s) {
       // a sample strictly inside the tile has this tile's piece only
       const int pb = s == s0 ? meta.pb0 : s == s1 ? meta.pb1 : meta.pbase + (s - s0);
@@ -522,6 +547,181 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
   }
 }
 
+// ------------------------------------------------------------------ fused bin permutation
+// The de-duplicated bin dispatch of Sec. 4.5 for the forward's own top-k, run at the end of the
+// forward by a group of warps per CTA (warps that are idle once the CTA's gate GEMM is done),
+// while the CTA's first epilogue warp reduces samples. Every CTA owns a contiguous run of tiles;
+// its epilogue warps add their rows' (token, bin) pairs into a shared total. The group publishes
+// the total; after a grid barrier (the launch is cooperative, so every CTA is resident) a CTA's
+// base in bin b is the pairs of all bins before b plus those of the CTAs before it in bin b, and
+// its tokens are placed in order with ballot ranks. Entries, offsets and counts equal those of
+// the standalone permutation kernel: pairs grouped by bin, by token inside a bin; dispatch and
+// expert counts are integer sums.
+__host__ __device__ inline size_t perm_scratch_ints(int E) {
+  return 7u * kMaxBins + static_cast<size_t>(kMaxBins) * kMaxBins + 2u * static_cast<size_t>(E) + 4u;
+}
+
+// One token's selection for the permutation: its experts with their bins and slot bits, its set
+// of bins, modality (0 vision, 1 text) and dispatch home (-1: invalid).
+template <int KM>
+struct PermSel {
+  int e[KM], b[KM];
+  uint32_t sbit[KM];
+  uint32_t bins;
+  int m, home;
+};
+
+template <int KM>
+__device__ __forceinline__ void perm_load_sel(const FwdParams& p, int j, PermSel<KM>& t) {
+  const Dims& dm = p.dm;
+  const FusedPerm& f = p.perm;
+  const bool valid = j < dm.T;
+  t.bins = 0u;
+  t.m = 0;
+  t.home = 0;
+#pragma unroll
+  for (int i = 0; i < KM; ++i) {
+    t.e[i] = -1;
+    t.b[i] = -1;
+    t.sbit[i] = 0u;
+    if (valid && i < dm.k) {
+      const int e = __ldcg(p.topk_idx + static_cast<size_t>(j) * dm.k + i);   // this CTA's rows
+      t.e[i] = e;
+      t.b[i] = dm.contig_bins ? e / dm.N_B : __ldg(p.ws.expert_bin + e);
+      t.sbit[i] = 1u << __ldg(p.ws.expert_slot + e);
+      t.bins |= 1u << t.b[i];
+    }
+  }
+  if (valid) {
+    t.m = (f.is_vision && !f.is_vision[j]) ? 1 : 0;
+    t.home = f.home ? f.home[j] : static_cast<int>((static_cast<long long>(j) * dm.K) / dm.T);
+    if (t.home < 0 || t.home >= dm.K) {
+      atomicOr(p.ws.status, kStatusData);
+      t.home = -1;
+    }
+  }
+}
+
+// gtid: the thread's index in the group (0 .. 32 nw - 1); bar_id: a named barrier for the group;
+// ctot: the CTA's pair counts per bin (complete at perm_go); scratch: perm_scratch_ints(E) ints of
+// shared memory that nothing else uses after perm_go.
+template <int KM>
+__device__ void perm_tail(const FwdParams& p, int t_beg, int t_end, int gtid, int nw, int bar_id,
+                          const int* ctot, int* scratch, uint64_t* perm_go, const WaitCtx& wc) {
+  const Dims& dm = p.dm;
+  const FusedPerm& f = p.perm;
+  const int K = dm.K, E = dm.E;
+  const int gs = nw * 32, gw = gtid >> 5, lane = gtid & 31;
+  int* wcnt = scratch;                          // [4][kMaxBins] per-warp counts, then their bases
+  int* base = wcnt + 4 * kMaxBins;              // [kMaxBins] next position of this CTA in bin b
+  int* pre_s = base + kMaxBins;                 // [kMaxBins]
+  int* tot_s = pre_s + kMaxBins;                // [kMaxBins]
+  int* disp = tot_s + kMaxBins;                 // [K][K] dispatch of this CTA's tokens
+  int* ecnt = disp + kMaxBins * kMaxBins;       // [2][E] expert counts of this CTA's tokens
+  int* flag = ecnt + 2 * E;
+  if (gtid == 0) *flag = mbar_wait(perm_go, 0, wc) ? 1 : 0;
+  named_bar(bar_id, gs);
+  if (!*flag) return;
+  // the first round's selections (they land while the other CTAs finish), then the CTA's counts
+  const int G = gridDim.x;
+  PermSel<KM> sel;
+  perm_load_sel<KM>(p, t_beg * kTileRows + gtid, sel);
+  if (gtid < K) f.cta_counts[gtid * G + blockIdx.x] = ctot[gtid];
+  for (int i = gtid; i < K * K; i += gs) disp[i] = 0;
+  for (int i = gtid; i < 2 * E; i += gs) ecnt[i] = 0;
+  if (blockIdx.x == 0) {                        // zeroed before any CTA passes the barrier
+    for (int i = gtid; i < K * K; i += gs) f.dispatch[i] = 0;
+    if (f.expert_counts)
+      for (int i = gtid; i < 2 * E; i += gs) f.expert_counts[i] = 0;
+  }
+  if (gtid < K || blockIdx.x == 0) __threadfence();
+  named_bar(bar_id, gs);
+  if (gtid == 0) *flag = grid_barrier(f.sync, G, p.limit_ns, p.ws.status) ? 1 : 0;
+  named_bar(bar_id, gs);
+  if (!*flag) return;
+
+  // this CTA's base in every bin
+  for (int kb = gw; kb < K; kb += nw) {
+    int pre = 0, tot = 0;
+    const int* row = f.cta_counts + kb * G;
+#pragma unroll 4
+    for (int c = lane; c < G; c += 32) {
+      const int v = __ldcg(row + c);
+      tot += v;
+      if (c < static_cast<int>(blockIdx.x)) pre += v;
+    }
+    pre = __reduce_add_sync(0xffffffffu, pre);
+    tot = __reduce_add_sync(0xffffffffu, tot);
+    if (lane == 0) {
+      pre_s[kb] = pre;
+      tot_s[kb] = tot;
+    }
+  }
+  named_bar(bar_id, gs);
+  if (gtid == 0) {
+    int run = 0;
+    for (int kb = 0; kb < K; ++kb) {
+      base[kb] = run + pre_s[kb];
+      if (blockIdx.x == 0) f.bin_offsets[kb] = run;
+      run += tot_s[kb];
+    }
+    if (blockIdx.x == 0) f.bin_offsets[K] = run;
+  }
+  named_bar(bar_id, gs);
+
+  // the CTA's tokens in order: per round, warp counts per bin -> bases over the group's warps ->
+  // ballot ranks inside the warp
+  const unsigned lt_mask = (1u << lane) - 1u;
+  bool first = true;
+  for (int tile = t_beg; tile < t_end; ++tile) {
+    for (int r0 = 0; r0 < kTileRows; r0 += gs) {
+      const int j = tile * kTileRows + r0 + gtid;
+      if (!first) perm_load_sel<KM>(p, j, sel);
+      first = false;
+      for (int kb = 0; kb < K; ++kb) {
+        const unsigned bal = __ballot_sync(0xffffffffu, (sel.bins >> kb) & 1u);
+        if (lane == 0) wcnt[gw * kMaxBins + kb] = __popc(bal);
+      }
+      named_bar(bar_id, gs);
+      if (gtid < K) {
+        int run = base[gtid];
+        for (int w = 0; w < nw; ++w) {
+          const int t = wcnt[w * kMaxBins + gtid];
+          wcnt[w * kMaxBins + gtid] = run;
+          run += t;
+        }
+        base[gtid] = run;
+      }
+      named_bar(bar_id, gs);
+      const unsigned same_home = __match_any_sync(0xffffffffu, sel.home);
+      for (int kb = 0; kb < K; ++kb) {
+        const unsigned bal = __ballot_sync(0xffffffffu, (sel.bins >> kb) & 1u);
+        if ((sel.bins >> kb) & 1u) {
+          const int pos = wcnt[gw * kMaxBins + kb] + __popc(bal & lt_mask);
+          uint32_t mask = 0u;
+#pragma unroll
+          for (int i = 0; i < KM; ++i) mask |= (sel.b[i] == kb) ? sel.sbit[i] : 0u;
+          f.perm_token[pos] = j;
+          f.perm_mask[pos] = mask;
+          const unsigned grp = bal & same_home;
+          if (sel.home >= 0 && lane == __ffs(grp) - 1) atomicAdd(&disp[sel.home * K + kb], __popc(grp));
+        }
+      }
+      if (f.expert_counts) {
+#pragma unroll
+        for (int i = 0; i < KM; ++i)
+          if (sel.e[i] >= 0) atomicAdd(&ecnt[sel.m * E + sel.e[i]], 1);
+      }
+      named_bar(bar_id, gs);                    // wcnt is rewritten by the next round
+    }
+  }
+  for (int i = gtid; i < K * K; i += gs)
+    if (disp[i]) atomicAdd(f.dispatch + i, disp[i]);
+  if (f.expert_counts)
+    for (int i = gtid; i < 2 * E; i += gs)
+      if (ecnt[i]) atomicAdd(f.expert_counts + i, ecnt[i]);
+}
+
 // ------------------------------------------------------------------ tcgen05 forward (bf16)
 
 __host__ __device__ inline size_t fwd_stage_bytes(int N) { return 16384u + static_cast<size_t>(N) * 128u; }
@@ -535,7 +735,7 @@ __host__ __device__ inline size_t fwd_smem_bytes(int N, int n_stages, int d, int
   if (stg) b += fwd_stg_bytes(E);
   if (gauss) b += 2u * sizeof(float) * static_cast<size_t>(round_up(d, kFwdBK));
   b += sizeof(float) * (epi_smem_floats(K) + 256u + 8u);
-  b += sizeof(uint64_t) * (2u * n_stages + 16u);
+  b += sizeof(uint64_t) * (2u * n_stages + 17u + kCoefBars);
   b += 16u;
   return b + 1024u;   // alignment slack
 }
@@ -555,6 +755,9 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   // same W tile from L2 at the same moment
   const int kb0 = blockIdx.x % n_kb;
   auto kb_at = [&](int i) { return (kb0 + i) % n_kb; };
+  // a contiguous run of tiles per CTA (the fused permutation orders its entries by CTA)
+  const int t_beg = static_cast<int>(static_cast<long long>(blockIdx.x) * p.n_tiles / gridDim.x);
+  const int t_end = static_cast<int>(static_cast<long long>(blockIdx.x + 1) * p.n_tiles / gridDim.x);
   const size_t sbytes = fwd_stage_bytes(N);
 
   uint8_t* q = base;
@@ -574,8 +777,10 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   uint64_t* drain = reinterpret_cast<uint64_t*>(q);     q += 8;
   uint64_t* bar_in = reinterpret_cast<uint64_t*>(q);    q += 8;
   uint64_t* bar_out = reinterpret_cast<uint64_t*>(q);   q += 8;
-  uint64_t* coef_bar = reinterpret_cast<uint64_t*>(q);  q += 8;
+  uint64_t* coef_bar = reinterpret_cast<uint64_t*>(q);  q += 8 * kCoefBars;
   uint64_t* coef_issued = reinterpret_cast<uint64_t*>(q);  q += 8;
+  uint64_t* gc_bar = reinterpret_cast<uint64_t*>(q);    q += 8;
+  uint64_t* perm_go = reinterpret_cast<uint64_t*>(q);   q += 8;
   uint64_t* stg_full = reinterpret_cast<uint64_t*>(q);  q += 8;
   uint64_t* stg_free = reinterpret_cast<uint64_t*>(q);  q += 8;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q); q += 4;
@@ -600,7 +805,12 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     mbar_init(bar_in, 128);
     mbar_init(bar_out, 128);
     mbar_init(coef_bar, 256);
+    for (int i = 1; i < kCoefBars; ++i) mbar_init(coef_bar + i, 128);
     mbar_init(coef_issued, 256);
+    mbar_init(gc_bar, 256);
+    mbar_init(perm_go, 1);
+    int* ctot = epi_smem(epi, dm.K, bar_in, bar_out).ctot;
+    for (int i = 0; i < kMaxBins; ++i) ctot[i] = 0;
     mbar_init(stg_full, 128);
     mbar_init(stg_free, 1);
     fence_mbar_init();
@@ -619,40 +829,69 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   pdl_trigger();
 
   if (kGauss && warp >= 2) {
-    // this CTA's Gaussian coefficients (eqs. 8-9), computed by the epilogue and Gaussian warps
-    // (256 threads) as feature pairs interleaved as float4 {ga[2i], ga[2i+1], gb[2i], gb[2i+1]};
-    // four pairs per thread and round, loads first; the first round is requested before the
-    // producer starts the X stream
-    const int ct = threadIdx.x - 64;
+    // this CTA's Gaussian coefficients (eqs. 8-9), float4 {ga[2i], ga[2i+1], gb[2i], gb[2i+1]}
+    // per feature pair i, computed in the order in which the CTA walks the K-blocks, in chunks
+    // of eight blocks (256 pairs): chunk 0 by the epilogue and Gaussian warps together, one pair
+    // per thread, so that the Gaussian warps consume the first stages early; the later chunks
+    // by the four epilogue warps, two pairs per thread, while the stream runs. The loads of
+    // chunks 0-3 are all issued before the producer starts the X stream.
+    const int ct = threadIdx.x - 64;            // 0..255; 0..127 in the epilogue warps
+    const bool epi_w = warp < 6;
     const float2* mu2 = reinterpret_cast<const float2*>(p.mu);
     const float2* var2 = reinterpret_cast<const float2*>(p.var);
     const int np = dm.d / 2;
+    const int n_pos = n_kb * 32;
+    const int n_chunks = (n_kb + 7) / 8;
+    auto pair_at = [&](int pos) { return kb_at(pos >> 5) * 32 + (pos & 31); };
+    auto load_pair = [&](int pos, float2 (&v)[4]) {
+      const int i = pos < n_pos ? pair_at(pos) : np;
+      const bool in = i < np;
+      v[0] = in ? __ldg(mu2 + i) : make_float2(0.f, 0.f);
+      v[1] = in ? __ldg(mu2 + np + i) : make_float2(0.f, 0.f);
+      v[2] = in ? __ldg(var2 + i) : make_float2(1.f, 1.f);
+      v[3] = in ? __ldg(var2 + np + i) : make_float2(1.f, 1.f);
+    };
     float part = 0.f;
-    bool announced = false;
-    for (int i0 = ct; i0 < dpad / 2; i0 += 4 * 256) {
-      float2 mv[4], mt[4], vv[4], vt[4];
+    auto store_pair = [&](int pos, const float2 (&v)[4]) {
+      if (pos < n_pos) part += gauss_coef_pair(v[0], v[1], v[2], v[3], cq + pair_at(pos));
+    };
+    constexpr int kPre = 3;                     // chunks 1..3: loads issued up front
+    float2 c0[4], pre[kPre][2][4];
+    load_pair(ct, c0);
+    if (epi_w) {
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const int i = i0 + 256 * u;
-        const bool in = i < np;
-        mv[u] = in ? __ldg(mu2 + i) : make_float2(0.f, 0.f);
-        mt[u] = in ? __ldg(mu2 + np + i) : make_float2(0.f, 0.f);
-        vv[u] = in ? __ldg(var2 + i) : make_float2(1.f, 1.f);
-        vt[u] = in ? __ldg(var2 + np + i) : make_float2(1.f, 1.f);
+      for (int c = 1; c <= kPre; ++c) {
+        load_pair(256 * c + ct, pre[c - 1][0]);
+        load_pair(256 * c + 128 + ct, pre[c - 1][1]);
       }
-      if (!announced) {
-        mbar_arrive(coef_issued);
-        announced = true;
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-        if (i0 + 256 * u < dpad / 2) part += gauss_coef_pair(mv[u], mt[u], vv[u], vt[u], cq + i0 + 256 * u);
     }
-    if (!announced) mbar_arrive(coef_issued);
+    mbar_arrive(coef_issued);
+    store_pair(ct, c0);
+    mbar_arrive(coef_bar);
+    if (epi_w) {
+      // chunk c completes barrier min(c, kCoefBars - 1); the last barrier covers every chunk
+      // from kCoefBars - 1 on and completes after the last one
+#pragma unroll
+      for (int c = 1; c <= kPre; ++c) {
+        if (c < n_chunks) {
+          store_pair(256 * c + ct, pre[c - 1][0]);
+          store_pair(256 * c + 128 + ct, pre[c - 1][1]);
+          if (c < kCoefBars - 1 || c == n_chunks - 1) mbar_arrive(coef_bar + min(c, kCoefBars - 1));
+        }
+      }
+      for (int c = kPre + 1; c < n_chunks; ++c) {
+        float2 v0[4], v1[4];
+        load_pair(256 * c + ct, v0);
+        load_pair(256 * c + 128 + ct, v1);
+        store_pair(256 * c + ct, v0);
+        store_pair(256 * c + 128 + ct, v1);
+        if (c < kCoefBars - 1 || c == n_chunks - 1) mbar_arrive(coef_bar + min(c, kCoefBars - 1));
+      }
+    }
     if (!isfinite(part)) atomicOr(p.ws.status, kStatusData);
     part = warp_sum(part);
     if (lane == 0) gred[warp - 2] = part;
-    mbar_arrive(coef_bar);
+    mbar_arrive(gc_bar);
   }
 
   if (warp == 0) {
@@ -665,7 +904,7 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       const uint32_t tx = static_cast<uint32_t>(sbytes);
       // the Gaussian statistics are requested before the X stream floods the memory system
       if (kGauss) ok = mbar_wait(coef_issued, 0, wc);
-      for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x) {
+      for (int tile = t_beg; tile < t_end && ok; ++tile) {
         for (int kb = 0; kb < n_kb; ++kb) {
           if (!mbar_wait(empty + st, ph ^ 1u, wc)) { ok = false; break; }
           uint8_t* xs = stage + st * sbytes;
@@ -693,7 +932,7 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       uint32_t ph = 0;
       int lt = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++lt) {
+      for (int tile = t_beg; tile < t_end && ok; ++tile, ++lt) {
         const int buf = lt & 1;
         const uint32_t use = static_cast<uint32_t>(lt >> 1);
         if (!mbar_wait(acc_empty + buf, (use & 1u) ^ 1u, wc)) { ok = false; break; }
@@ -724,6 +963,7 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     const int lg = warp & 3;                 // TMEM lane group accessible to this warp
     const int row = lg * 32 + lane;          // tile row == TMEM lane == token offset
     EpiSmem es = epi_smem(epi, dm.K, bar_in, bar_out);
+    es.perm_go = perm_go;
     if (use_stg) {
       es.stg = stg;
       es.stg_full = stg_full;
@@ -747,9 +987,14 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       __device__ void operator()() const { tc_fence_before(); mbar_arrive(bar); }
     };
     const uint32_t tl = tmem_base + (static_cast<uint32_t>(lg * 32) << 16);
+    float gc = 0.f;                          // constant term of eq. (8), -1/2 sum of the parts
+    if (kGauss && mbar_wait(gc_bar, 0, wc)) {
+      for (int w = 0; w < 8; ++w) gc += gred[w];
+      gc *= -0.5f;
+    }
     uint32_t n_in = 0;
     int lt = 0;
-    for (int tile = blockIdx.x; tile < p.n_tiles; tile += gridDim.x, ++lt) {
+    for (int tile = t_beg; tile < t_end; ++tile, ++lt) {
       const int buf = lt & 1;
       const uint32_t use = static_cast<uint32_t>(lt >> 1);
       const TileMeta meta = load_tile_meta(p, tile, row);    // lands while the tile streams in
@@ -758,11 +1003,11 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       float dll = 0.f;
       if (kGauss) {
         if (!mbar_wait(g_full + buf, use & 1u, wc)) break;
-        dll = dll_s[buf * 128 + row];
+        dll = dll_s[buf * 128 + row] + gc;
         mbar_arrive(g_empty + buf);
       }
       epilogue_tile<KM>(p, Src{tl + static_cast<uint32_t>(buf * N), dm.E}, Rel{acc_empty + buf},
-                        tile, row, lt, dll, meta, es, wc, n_in);
+                        tile, row, lt, dll, meta, es, wc, n_in, tile == t_end - 1);
     }
     if (use_stg && row == 0) tma_store_wait_all<0>();   // the score stores complete before exit
   } else {
@@ -774,17 +1019,14 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     if (kGauss) {
       const int gw = warp - 6;
       const int gt = gw * 32 + lane;
-      bool ok = mbar_wait(coef_bar, 0, wc);
-      float gc = 0.f;
-      for (int w = 0; w < 8; ++w) gc += gred[w];
-      gc *= -0.5f;
+      bool ok = true;
       // byte offset of this lane's word inside a 128-byte swizzled row r: chunk (l/4) ^ (r & 7)
       const uint32_t wcol = static_cast<uint32_t>(lane & 3) * 4u;
       const uint32_t chk = static_cast<uint32_t>(lane >> 2);
       int st = 0;
       uint32_t ph = 0;
       int lt = 0;
-      for (int tile = blockIdx.x; tile < p.n_tiles && ok; tile += gridDim.x, ++lt) {
+      for (int tile = t_beg; tile < t_end && ok; ++tile, ++lt) {
         const int buf = lt & 1;
         const uint32_t use = static_cast<uint32_t>(lt >> 1);
         if (!mbar_wait(g_empty + buf, (use & 1u) ^ 1u, wc)) break;
@@ -792,6 +1034,9 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
 #pragma unroll
         for (int r = 0; r < 32; ++r) acc[r] = 0.f;
         for (int kb = 0; kb < n_kb; ++kb) {
+          // the coefficients of this block's chunk (complete for every later tile)
+          if (lt == 0 && (kb & 7) == 0 && kb < 8 * kCoefBars &&
+              !mbar_wait(coef_bar + (kb >> 3), 0, wc)) { ok = false; break; }
           if (!mbar_wait(full + st, ph, wc)) { ok = false; break; }
           const uint8_t* xs = stage + st * sbytes + gw * 32 * 128;
           const float4 cf = cq[kb_at(kb) * 32 + lane];
@@ -807,10 +1052,18 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
           if (++st == n_stages) { st = 0; ph ^= 1u; }
         }
         if (!ok) break;
-        dll_s[buf * 128 + gt] = warp_transpose_sum(acc) + gc;
+        dll_s[buf * 128 + gt] = warp_transpose_sum(acc);
         mbar_arrive(g_full + buf);
       }
     }
+  }
+  // the fused permutation, by the Gaussian warps (without them, the producer and MMA warps)
+  // once their part of the CTA's tiles is done; the stage buffers are free after perm_go
+  if (p.perm.perm_token) {
+    int* ps = reinterpret_cast<int*>(stage);
+    const int* ctot = epi_smem(epi, dm.K, bar_in, bar_out).ctot;
+    if (kGauss && warp >= 6) perm_tail<KM>(p, t_beg, t_end, threadIdx.x - 192, 4, 1, ctot, ps, perm_go, wc);
+    if (!kGauss && warp < 2) perm_tail<KM>(p, t_beg, t_end, threadIdx.x, 2, 1, ctot, ps, perm_go, wc);
   }
 
   tc_fence_before();
@@ -923,8 +1176,8 @@ k_router_fwd_f32(const FwdParams p) {
     WaitCtx wc{abort_flag, p.ws.status, p.limit_ns};
     const EpiSmem es = epi_smem(epi, dm.K, bars + 0, bars + 1);
     uint32_t n_in = 0;
-    const TileMeta meta = load_tile_meta(p, tile, t);
-    epilogue_tile<KM>(p, src, rel, tile, t, 0, kGauss ? dll_s[t] : 0.f, meta, es, wc, n_in);
+    const TileMeta meta = load_tile_meta(p, tile, t);   // (no fused permutation on this path)
+    epilogue_tile<KM>(p, src, rel, tile, t, 0, kGauss ? dll_s[t] : 0.f, meta, es, wc, n_in, true);
   }
 }
 
@@ -956,6 +1209,8 @@ cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
   const int n_stages = stages_for(use_stg);
   const size_t smem = fwd_smem_bytes(N, n_stages, p.dm.d, p.dm.K, p.dm.E, gauss, use_stg);
   if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
+  if (p.perm.perm_token && static_cast<size_t>(n_stages) * fwd_stage_bytes(N) < sizeof(int) * perm_scratch_ints(p.dm.E))
+    return cudaErrorInvalidConfiguration;
   const int grid = p.n_tiles < n_sms ? p.n_tiles : n_sms;
   const CUtensorMap& tg = use_stg ? *tmG : tmX;           // unused without staging
   return dispatch_km(p.dm.k, [&](auto km) -> cudaError_t {
@@ -963,8 +1218,23 @@ cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
     auto k = gauss ? k_router_fwd_tc<true, KM> : k_router_fwd_tc<false, KM>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(k, dim3(grid), dim3(gauss ? 320 : 192), smem, s, tmX, tmW, tg, p, N, n_stages,
-                      use_stg ? 1 : 0);
+    if (!p.perm.perm_token)
+      return launch_pdl(k, dim3(grid), dim3(gauss ? 320 : 192), smem, s, tmX, tmW, tg, p, N, n_stages,
+                        use_stg ? 1 : 0);
+    // the fused permutation has a grid barrier: every CTA must be resident (cooperative launch)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(gauss ? 320 : 192);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, k, tmX, tmW, tg, p, N, n_stages, use_stg ? 1 : 0);
   });
 }
 

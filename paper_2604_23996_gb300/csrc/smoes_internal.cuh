@@ -58,6 +58,20 @@ struct Dims {
   int contig_bins;           // bin b holds experts [b N_B, (b+1) N_B) and N_B % 4 == 0
 };
 
+// The bin permutation of the forward's own top-k, done inside the forward launch (Sec. 4.5);
+// perm_token == null: not requested.
+struct FusedPerm {
+  const int32_t* home;       // [T] or null (contiguous split)
+  const uint8_t* is_vision;  // [T] (required with expert_counts)
+  int32_t* bin_offsets;
+  int32_t* perm_token;
+  uint32_t* perm_mask;
+  int32_t* dispatch;
+  int32_t* expert_counts;
+  int32_t* cta_counts;       // [K][G] pairs of each bin in each CTA's tiles (workspace)
+  uint32_t* sync;            // [2] grid barrier words (workspace, zero between calls)
+};
+
 struct FwdParams {
   Dims dm;
   WsView ws;
@@ -74,6 +88,7 @@ struct FwdParams {
   float* joint;
   float* mi;
   float* loss;
+  FusedPerm perm;
   int n_tiles;
   uint64_t limit_ns;
 };

@@ -98,25 +98,29 @@ def to_dev(wl, dev):
 
 
 def run_gpu(wl, bd, mode="gauss", M_in=None, d_topk_w=None, loss_scale=1.0, want_dx=True,
-            want_dlogits=True, home=None, dev="cuda"):
-    """One forward + backward + permutation through the C ABI; returns numpy outputs."""
+            want_dlogits=True, home=None, dev="cuda", fused=False):
+    """One forward + backward + permutation through the C ABI; returns numpy outputs.
+    fused: the permutation is requested from the forward call (smoes_router_fwd_permute)."""
     dtype = bd.SMOES_BF16 if wl.dtype == torch.bfloat16 else bd.SMOES_F32
     r = bd.Router(wl.T, wl.d, wl.E, wl.k, wl.n_bins, wl.sample_offsets, wl.expert_bin, dtype,
                   renorm_topk=wl.renorm_topk)
     X, W, mu, var = to_dev(wl, dev)
+    hv = None if home is None else torch.as_tensor(home, dtype=torch.int32).to(dev)
+    isv = torch.from_numpy(wl.is_vision).to(dev)
+    fwd = (lambda **kw: r.forward_permute(is_vision=isv, home=hv, **kw)) if fused else r.forward
     if mode == "gauss":
-        r.forward(X, W, mu=mu, var=var, tau=wl.tau)
+        fwd(X=X, W=W, mu=mu, var=var, tau=wl.tau)
         M = r.M
     else:
         M = torch.as_tensor(M_in, dtype=torch.float32).to(dev).contiguous()
-        r.forward(X, W, M_in=M)
+        fwd(X=X, W=W, M_in=M)
     dW = torch.full((wl.E, wl.d), float("nan"), dtype=torch.float32, device=dev)
     dX = torch.empty_like(X) if want_dx else None
     dl = torch.empty((wl.T, wl.E), dtype=torch.float32, device=dev) if want_dlogits else None
     dtw = None if d_topk_w is None else torch.as_tensor(d_topk_w, dtype=torch.float32).to(dev)
     r.backward(X, W, M, dW, dX=dX, dlogits=dl, loss_scale=loss_scale, d_topk_w=dtw)
-    hv = None if home is None else torch.as_tensor(home, dtype=torch.int32).to(dev)
-    r.permute(is_vision=torch.from_numpy(wl.is_vision).to(dev), home=hv)
+    if not fused:
+        r.permute(is_vision=isv, home=hv)
     code, n_absent = r.device_status()
     torch.cuda.synchronize()
     P = int(r.bin_offsets[-1].item())
@@ -149,7 +153,7 @@ def run_oracle(wl, mode="gauss", M_in=None, loss_scale=1.0, d_topk_w=None, topk_
     return dict(M=M, fwd=fwd, dz=dz, dW=dz.T @ Xd, dX=dz @ Wd)
 
 
-def compare(wl, g, ref, check_dx=True):
+def compare(wl, g, ref, check_dx=True, home=None):
     """Element-by-element comparison; returns a dict of measured errors and excluded counts."""
     res = {}
     fwd = ref["fwd"]
@@ -172,7 +176,7 @@ def compare(wl, g, ref, check_dx=True):
         else:
             res["dX"] = assert_tensor_close(g["dX"], ref["dX"], "dX")
     # permutation, stage-wise: the oracle permutes the GPU's own top-k, bit for bit
-    pr = O.bin_permute(g["topk_idx"], wl.expert_bin, wl.n_bins, is_vision=wl.is_vision)
+    pr = O.bin_permute(g["topk_idx"], wl.expert_bin, wl.n_bins, home=home, is_vision=wl.is_vision)
     np.testing.assert_array_equal(g["offsets"], pr["offsets"], err_msg="bin_offsets")
     np.testing.assert_array_equal(g["perm"], pr["perm"], err_msg="perm_token")
     np.testing.assert_array_equal(g["mask"].astype(np.uint64), pr["mask"], err_msg="perm_mask")

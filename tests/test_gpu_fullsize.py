@@ -48,22 +48,26 @@ class _Acc:
         return r
 
 
-def _run_full(bd, wl, M_in=None):
+def _run_full(bd, wl, M_in=None, fused=True):
+    """fused: the permutation comes from the forward call, as bench.py runs the step."""
     dev = "cuda"
     dt = bd.SMOES_BF16 if wl.dtype == torch.bfloat16 else bd.SMOES_F32
     r = bd.Router(wl.T, wl.d, wl.E, wl.k, wl.n_bins, wl.sample_offsets, wl.expert_bin, dt)
     X, W = wl.X.to(dev), wl.W.to(dev)
+    isv = torch.from_numpy(wl.is_vision).to(dev)
+    fwd = (lambda **kw: r.forward_permute(is_vision=isv, **kw)) if fused else r.forward
     if M_in is None:
-        r.forward(X, W, mu=wl.mu.to(dev), var=wl.var.to(dev), tau=wl.tau)
+        fwd(X=X, W=W, mu=wl.mu.to(dev), var=wl.var.to(dev), tau=wl.tau)
         M = r.M
     else:
         M = torch.from_numpy(M_in).to(dev)
-        r.forward(X, W, M_in=M)
+        fwd(X=X, W=W, M_in=M)
     dW = torch.empty((wl.E, wl.d), dtype=torch.float32, device=dev)
     dX = torch.empty_like(X)
     dl = torch.empty((wl.T, wl.E), dtype=torch.float32, device=dev)
     r.backward(X, W, M, dW, dX=dX, dlogits=dl, loss_scale=1.0)
-    r.permute(is_vision=torch.from_numpy(wl.is_vision).to(dev))
+    if not fused:
+        r.permute(is_vision=isv)
     assert r.device_status()[0] == 0
     torch.cuda.synchronize()
     n = int(r.bin_offsets[-1].item())
@@ -128,6 +132,15 @@ def test_fullsize_router(bd, key):
     g = _run_full(bd, wl)
     excl = _check_per_sample(wl, g)
     print(f"{key}: T={wl.T} tie-excluded tokens {excl}")
+
+
+def test_fullsize_fused_equals_separate(bd):
+    # 256 tiles on at most 152 CTAs: CTAs with two tiles; every output bit for bit
+    wl = config_workload("small_hidden")
+    a = _run_full(bd, wl, fused=True)
+    b = _run_full(bd, wl, fused=False)
+    for key in a:
+        np.testing.assert_array_equal(np.asarray(a[key]), np.asarray(b[key]), err_msg=key)
 
 
 def test_fullsize_aligned_variant(bd):

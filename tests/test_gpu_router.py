@@ -73,6 +73,41 @@ def test_hard_labels_with_text_only_sample(bd):
     assert g["mi"][1] == 0.0
 
 
+@pytest.mark.parametrize("name", list(CASES))
+def test_fused_permute_parity(bd, name):
+    # smoes_router_fwd_permute: forward outputs and the permutation of its own top-k (one launch
+    # on bf16 plans, two calls on fp32) against the oracle
+    seed, T, d, E, k, K, lens, dt, aligned = CASES[name]
+    wl = random_router_case(seed, T, d, E, k, K, lens, dtype=dt, aligned=aligned)
+    g = run_gpu(wl, bd, mode="gauss", loss_scale=0.7, fused=True)
+    ref = run_oracle(wl, mode="gauss", loss_scale=0.7)
+    compare(wl, g, ref)
+
+
+def test_fused_permute_provided_scores_custom_home(bd):
+    # without the Gaussian warps the producer and MMA warps run the permutation; non-consecutive
+    # bins and a custom dispatch home
+    wl = random_router_case(27, 1500, 192, 48, 5, 6, [200, 1100, 200], aligned=True)
+    rng = np.random.default_rng(1)
+    wl.expert_bin = rng.permutation(wl.expert_bin).astype(np.int32)
+    Mv = rng.uniform(0.02, 0.98, wl.T)
+    M = np.stack([Mv, 1 - Mv], 1).astype(np.float32)
+    home = (np.arange(wl.T) * 5) % wl.n_bins
+    g = run_gpu(wl, bd, mode="provided", M_in=M, home=home, fused=True)
+    ref = run_oracle(wl, mode="provided", M_in=M.astype(np.float64))
+    compare(wl, g, ref, home=home)
+
+
+def test_fused_permute_equals_separate_calls(bd):
+    wl = random_router_case(26, 2000, 256, 64, 6, 8, [700, 1300], aligned=True)
+    a = run_gpu(wl, bd, mode="gauss")
+    b = run_gpu(wl, bd, mode="gauss", fused=True)
+    for key in a:
+        if a[key] is None:
+            continue
+        np.testing.assert_array_equal(np.asarray(a[key]), np.asarray(b[key]), err_msg=key)
+
+
 def test_custom_home_dispatch(bd):
     wl = random_router_case(23, 640, 128, 32, 4, 4, [320, 320], aligned=True)
     home = (np.arange(wl.T) * 7) % wl.n_bins
