@@ -329,10 +329,11 @@ def main():
                 part_graphs.append(g)
     torch.cuda.current_stream().wait_stream(s)
     torch.cuda.synchronize()
-    # our kernels per step: attention 1; fwd + permutation 2 (forward, scatter; fp32: Gaussian
-    # coefficients 1, forward 1, permutation 1); bwd 3 (dz prep, main, dW reduce; fp32: main, dW reduce)
+    # our kernels per step: attention 1; fwd + permutation 1 (one cooperative launch; fp32:
+    # Gaussian coefficients 1, forward 1, permutation 1); bwd 3 (dz prep, main, dW reduce; fp32:
+    # main, dW reduce)
     f32 = dtype != bd.SMOES_BF16
-    fwd_launches = ((0 if use_attn else 1) + 2) if f32 else 2
+    fwd_launches = ((0 if use_attn else 1) + 2) if f32 else 1
     launches_per_step = (1 if use_attn else 0) + fwd_launches + (2 if f32 else 3)
 
     def step_timed():
