@@ -23,7 +23,7 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
   size_t status, sample_ticket, loss_ticket, offsets, token_sample, expert_bin, expert_slot,
-      piece_base, sample_pieces, pieces, mi32, tabs, gsave, dw_part, dz_img, perm, attn_ticket, attn_part,
+      piece_base, sample_pieces, pieces, mi32, tabs, gsave, ginv, dw_part, dz_img, perm, attn_ticket, attn_part,
       gcoef, perm_sync, fperm;
   size_t header_bytes;   // [0, header_bytes) is cleared by smoes_workspace_init
   size_t total;
@@ -68,6 +68,7 @@ WsView make_view(const smoes_plan_s* P, void* ws) {
   v.mi32 = reinterpret_cast<float*>(b + L.mi32);
   v.tabs = reinterpret_cast<float*>(b + L.tabs);
   v.gsave = reinterpret_cast<float*>(b + L.gsave);
+  v.ginv = reinterpret_cast<float*>(b + L.ginv);
   v.dw_part = reinterpret_cast<float*>(b + L.dw_part);
   v.dz_img = b + L.dz_img;
   v.perm_scratch = reinterpret_cast<int32_t*>(b + L.perm);
@@ -344,6 +345,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.mi32 = take(sizeof(float) * std::max(B, 1));
   L.tabs = take(sizeof(float) * 3 * K * static_cast<size_t>(std::max(B, 1)));
   L.gsave = take(sizeof(float) * static_cast<size_t>(T) * E);
+  L.ginv = take(sizeof(float) * static_cast<size_t>(std::max(T, 1)));
   L.dw_part = take(sizeof(float) * static_cast<size_t>(P->bwd_groups) * E * d.d);
   L.dz_img = take(d.dtype == SMOES_BF16 && E <= 128
                       ? static_cast<size_t>(P->bwd_tiles) * 2 * round_up(E, 64) * 128 : 0);

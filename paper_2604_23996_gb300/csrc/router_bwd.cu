@@ -44,6 +44,7 @@ __device__ __forceinline__ void load_upstream(const BwdParams& p, int j, Upstrea
   float gsel[kMaxTopK], d[kMaxTopK];
   float G = 0.f, dw = 0.f;
   const float* g = p.ws.gsave + static_cast<size_t>(j) * p.dm.E;
+  const float ginv = p.ws.ginv[j];
 #pragma unroll
   for (int i = 0; i < kMaxTopK; ++i) {
     u.idx[i] = -1;
@@ -54,7 +55,7 @@ __device__ __forceinline__ void load_upstream(const BwdParams& p, int j, Upstrea
       u.idx[i] = p.topk_idx[static_cast<size_t>(j) * k + i];
       d[i] = p.d_topk_w[static_cast<size_t>(j) * k + i];
       const int e = u.idx[i];
-      gsel[i] = (e >= 0 && e < p.dm.E) ? g[e] : 0.f;
+      gsel[i] = (e >= 0 && e < p.dm.E) ? g[e] * ginv : 0.f;
       G += gsel[i];
     }
   }
@@ -105,6 +106,7 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
   float g[8], u[8];
   if (valid) {
     const float* grow = p.ws.gsave + static_cast<size_t>(j) * E;
+    const float ginv = __ldcg(p.ws.ginv + j);
     if ((E & 3) == 0 && e0 + 8 <= E) {
       const float4 a = __ldcg(reinterpret_cast<const float4*>(grow + e0));
       const float4 b = __ldcg(reinterpret_cast<const float4*>(grow + e0 + 4));
@@ -113,6 +115,8 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
 #pragma unroll
       for (int q = 0; q < 8; ++q) g[q] = (e0 + q < E) ? __ldcg(grow + e0 + q) : 0.f;
     }
+#pragma unroll
+    for (int q = 0; q < 8; ++q) g[q] *= ginv;                 // the softmax score g_je
     const float2 m = __ldg(reinterpret_cast<const float2*>(p.M) + j);
     const float dv = m.x - 0.5f, dt = m.y - 0.5f;
     // the sample's coefficient table was written by the forward kernel and is read-only here
@@ -472,11 +476,12 @@ k_router_bwd_f32(const BwdParams p) {
     const bool has_up = valid && p.d_topk_w != nullptr;
     if (has_up) load_upstream(p, j, up);
     const float* g = p.ws.gsave + static_cast<size_t>(valid ? j : 0) * E;
+    const float ginv = valid ? p.ws.ginv[j] : 0.f;
     float part = 0.f;
     for (int e = qd; e < E; e += 4) {
       if (valid) {
         const int b = p.ws.expert_bin[e];
-        part += g[e] * (tb[2 * K + b] + dv * tb[b] + dt * tb[K + b]);
+        part += g[e] * ginv * (tb[2 * K + b] + dv * tb[b] + dt * tb[K + b]);
       }
     }
     part += __shfl_xor_sync(0xffffffffu, part, 1);
@@ -486,8 +491,9 @@ k_router_bwd_f32(const BwdParams p) {
       if (valid) {
         const int b = p.ws.expert_bin[e];
         const float u = tb[2 * K + b] + dv * tb[b] + dt * tb[K + b];
-        v = p.scale * g[e] * (u - part);
-        if (has_up) v += g[e] * (upstream_at(up, k, e) - up.gdt);
+        const float ge = g[e] * ginv;
+        v = p.scale * ge * (u - part);
+        if (has_up) v += ge * (upstream_at(up, k, e) - up.gdt);
         if (p.dlogits) p.dlogits[static_cast<size_t>(j) * E + e] = v;
       }
       dzs[r * (E + 1) + e] = v;

@@ -102,8 +102,13 @@ __device__ __forceinline__ float warp_transpose_sum(float (&v)[32]) {
 // every term a log1p of a small, directly computed quantity; h_k is formed from second-order
 // differences directly as well (see below). `red` is kMaxNV floats of shared scratch; the
 // sample's pieces [pb, pe) and token count n are passed in when already loaded (pb < 0: load).
+//
+// dry: the same instruction path with every global access and fence skipped. The first epilogue
+// warp runs it once while it waits for its first accumulator, so that this code, which a CTA
+// otherwise runs once at the very end, is in the instruction cache when the last piece of a
+// sample arrives (a dry run must not touch memory: its loads would queue behind the X stream).
 __device__ __noinline__ void sample_reduce(const FwdParams& p, int s, float* red, int pb, int pe,
-                                           int nt) {
+                                           int nt, bool dry) {
   const Dims& dm = p.dm;
   const int K = dm.K;
   const int NV = piece_values(K);
@@ -113,33 +118,23 @@ __device__ __noinline__ void sample_reduce(const FwdParams& p, int s, float* red
     pe = p.ws.sample_pieces[s + 1];
     nt = p.ws.offsets[s + 1] - p.ws.offsets[s];
   }
-  // value blocks c, c+1 (values 32c .. 32c+63): lane l loads the blocks of piece q0 + l, a
-  // butterfly sums the 32 pieces of each block, rounds of 32 pieces are added in order
+  // lane l sums value 32c + l over the sample's pieces in piece order, 16 loads in flight
 #pragma unroll 1
-  for (int c = 0; c * 32 < NV; c += 2) {
-    float acc0 = 0.f, acc1 = 0.f;
+  for (int c = 0; c * 32 < NV; ++c) {
+    const int v = 32 * c + lane;
+    const bool in = v < NV;
+    float acc = 0.f;
 #pragma unroll 1
-    for (int q0 = pb; q0 < pe; q0 += 32) {
-      float v0[32], v1[32];
-      const int q = q0 + lane;
-      const float* src = p.ws.pieces + static_cast<size_t>(q) * dm.pstride + 32 * c;
+    for (int q0 = pb; q0 < pe; q0 += 16) {
+      const float* src = p.ws.pieces + static_cast<size_t>(q0) * dm.pstride + (in ? v : 0);
+      float t[16];
 #pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        float4 f = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (q < pe && 32 * c + 4 * i < dm.pstride) f = __ldcg(reinterpret_cast<const float4*>(src + 4 * i));
-        float* v = i < 8 ? v0 + 4 * i : v1 + 4 * (i - 8);
-        v[0] = f.x; v[1] = f.y; v[2] = f.z; v[3] = f.w;
-      }
+      for (int i = 0; i < 16; ++i)
+        t[i] = (in && !dry && q0 + i < pe) ? __ldcg(src + static_cast<size_t>(i) * dm.pstride) : 0.f;
 #pragma unroll
-      for (int i = 0; i < 32; ++i) {           // row padding past the values
-        if (32 * c + i >= NV) v0[i] = 0.f;
-        if (32 * c + 32 + i >= NV) v1[i] = 0.f;
-      }
-      acc0 += warp_transpose_sum(v0);
-      if (32 * c + 32 < NV) acc1 += warp_transpose_sum(v1);
+      for (int i = 0; i < 16; ++i) acc += t[i];
     }
-    if (32 * c + lane < NV) red[32 * c + lane] = acc0;
-    if (32 * c + 32 + lane < NV) red[32 * c + 32 + lane] = acc1;
+    if (in) red[v] = acc;
   }
   __syncwarp();
   const bool act = lane < K;
@@ -195,7 +190,7 @@ __device__ __noinline__ void sample_reduce(const FwdParams& p, int s, float* red
     Pv = has_v ? P1 : 0.f;
     Pt = has_t ? P1 : 0.f;
   }
-  if (act) {
+  if (act && !dry) {
     float* tb = p.ws.tabs + static_cast<size_t>(s) * 3 * K;
     tb[lane] = a;
     tb[K + lane] = b;
@@ -205,7 +200,7 @@ __device__ __noinline__ void sample_reduce(const FwdParams& p, int s, float* red
       p.joint[(static_cast<size_t>(s) * 2 + 1) * K + lane] = Pt;
     }
   }
-  if (lane == 0) {
+  if (lane == 0 && !dry) {
     p.mi[s] = I;
     p.ws.mi32[s] = I;
     const uint32_t absent = (has_v ? 0u : 1u) + (has_t ? 0u : 1u);
@@ -213,17 +208,17 @@ __device__ __noinline__ void sample_reduce(const FwdParams& p, int s, float* red
     if (!isfinite(I) || !(sumQ > 0.f)) atomicOr(p.ws.status, kStatusData);
     p.ws.sample_ticket[s] = 0u;                       // ready for the next call
   }
-  __threadfence();
+  if (!dry) __threadfence();
   __syncwarp();
   uint32_t last = 0;
-  if (lane == 0) last = (atomicAdd(p.ws.loss_ticket, 1u) + 1u == static_cast<uint32_t>(dm.B));
+  if (lane == 0) last = dry || (atomicAdd(p.ws.loss_ticket, 1u) + 1u == static_cast<uint32_t>(dm.B));
   last = __shfl_sync(0xffffffffu, last, 0);
   if (last) {                                         // eq. (15) for one layer
-    __threadfence();
+    if (!dry) __threadfence();
     float t = 0.f;
-    for (int i = lane; i < dm.B; i += 32) t += __ldcg(p.ws.mi32 + i);
+    for (int i = lane; i < dm.B; i += 32) t += dry ? 0.f : __ldcg(p.ws.mi32 + i);
     t = warp_sum(t);
-    if (lane == 0) {
+    if (lane == 0 && !dry) {
       *p.loss = -t / static_cast<float>(dm.B);
       *p.ws.loss_ticket = 0u;
     }
@@ -257,73 +252,110 @@ __device__ __forceinline__ TileMeta load_tile_meta(const FwdParams& p, int tile,
   return m;
 }
 
-// Shared memory of the per-tile epilogue group (128 threads, one token row each; each warp
-// reads and writes only its own 32 rows of p_s and m_s).
+// Shared memory of the per-tile epilogue: two groups of 128 threads, one token row per thread in
+// each group (thread `row` of both groups owns tile row `row`); the groups split the logit
+// columns. Each warp reads and writes only its own 32 rows of the row tables.
 struct EpiSmem {
   float* p_s;            // [K][kPsStride] bin probabilities of the tile's rows
   float* m_s;            // [5][kPsStride] (M_v - 1/2, M_t - 1/2, M_v, M_t, 1) of the tile's rows
-  float* wpart;          // [2][4][kMaxNV] per-warp partial piece sums (double buffer)
-  float* red;            // [kMaxNV] sample-reduce scratch of the group's first warp
+  float* wpart;          // [2][4][kMaxNV] per-lane-quarter partial piece sums (double buffer)
+  float* red;            // [kMaxNV] sample-reduce scratch of the first warp
   int* ctot;             // [kMaxBins] (token, bin) pairs of the CTA's tiles (fused permutation)
-  uint64_t* bar_in;      // count 128: the warps' partials of one (tile, sample) are written
-  uint64_t* bar_out;     // count 128: the tile's pieces are written
+  float* xmax;           // [2][128] per-group row maxima of the logits
+  float* xsum;           // [2][128] per-group row sums of exp(z - max)
+  float* xtk;            // [kMaxTopK][128] group 1's top-k keys of each row
+  uint64_t* bar_in;      // count 256: the partials of one (tile, sample) are written
+  uint64_t* bar_out;     // count 256: the tile's pieces are written
+  uint64_t* xbar;        // [3] count 256: row maxima and keys / row sums / row tables exchanged
   uint64_t* perm_go;     // count 1: the CTA's top-k and pair counts are complete
-  // optional staging of the tile's softmax scores for one coalesced TMA store: 32-column blocks
-  // of [128 rows][128 bytes], 16-byte chunks swizzled by row (the 128-byte TMA swizzle)
+  // optional staging of the tile's scores for coalesced TMA stores: 32-column blocks of
+  // [128 rows][128 bytes], 16-byte chunks swizzled by row (the 128-byte TMA swizzle); each
+  // group stages and stores its own blocks
   uint8_t* stg;          // null: scores are stored row by row
-  uint64_t* stg_full;    // count 128: all rows staged
-  uint64_t* stg_free;    // count 1: the previous tile's store has read the staging
+  uint64_t* stg_full;    // [2] count 128: a group's rows are staged
+  uint64_t* stg_free;    // [2] count 1: a group's previous store has read the staging
   const CUtensorMap* tmG;
 };
 
 __host__ __device__ inline size_t epi_smem_floats(int K) {
-  return static_cast<size_t>(K) * kPsStride + 5u * kPsStride + 2u * 4u * kMaxNV + kMaxNV + kMaxBins;
+  return static_cast<size_t>(K) * kPsStride + 5u * kPsStride + 2u * 4u * kMaxNV + kMaxNV + kMaxBins +
+         4u * 128u + static_cast<size_t>(kMaxTopK) * 128u;
 }
 
-__device__ inline EpiSmem epi_smem(float* base, int K, uint64_t* bar_in, uint64_t* bar_out) {
+__device__ inline EpiSmem epi_smem(float* base, int K, uint64_t* bars) {
   EpiSmem es;
   es.p_s = base;
   es.m_s = es.p_s + K * kPsStride;
   es.wpart = es.m_s + 5 * kPsStride;
   es.red = es.wpart + 2 * 4 * kMaxNV;
   es.ctot = reinterpret_cast<int*>(es.red + kMaxNV);
-  es.bar_in = bar_in;
-  es.bar_out = bar_out;
+  es.xmax = es.red + kMaxNV + kMaxBins;
+  es.xsum = es.xmax + 256;
+  es.xtk = es.xsum + 256;
+  es.bar_in = bars;
+  es.bar_out = bars + 1;
+  es.xbar = bars + 2;
   es.perm_go = nullptr;
   es.stg = nullptr;
   es.stg_full = es.stg_free = nullptr;
   es.tmG = nullptr;
   return es;
 }
+constexpr int kEpiBars = 5;   // bar_in, bar_out, xbar[3]
 
-// Per-tile epilogue. Src::load16(c, v) returns logits [16c, 16c+16) of this thread's row,
-// -FLT_MAX past E (finite, so that its top-k key is not a NaN; warp-collective); release() is
-// called after the last logit read. row: token row in
-// the tile (0..127, the thread's index in the group); lt: index of the tile among those this
-// group processes; meta: the tile's metadata (load_tile_meta); n_in: completed phases of
-// bar_in (identical in all 128 threads). With the fused permutation every warp adds its rows'
-// (token, bin) pairs to es.ctot, and after the CTA's last tile the first warp arrives on
-// es.perm_go once all rows are counted.
+__device__ inline void init_epi_bars(uint64_t* bars) {
+  for (int i = 0; i < kEpiBars; ++i) mbar_init(bars + i, 256);
+}
+
+// Column split of the logits between the two epilogue groups: group 0 takes the 16-column chunks
+// [0, nc0), group 1 [nc0, nch). nc0 is even (32-column staging blocks stay in one group) and,
+// with consecutive bins, a multiple of N_B columns (no bin straddles the groups); otherwise
+// group 0 takes every column.
+__device__ __forceinline__ int epi_split(const Dims& dm) {
+  const int nch = (dm.E + 15) >> 4;
+  const int nc0 = 2 * ((nch + 3) >> 2);
+  if (nc0 >= nch || !dm.contig_bins || (16 * nc0) % dm.N_B != 0) return nch;
+  return nc0;
+}
+
+// Per-tile epilogue, run by both groups (grp 0, 1) for every tile. Src::load16(c, v) returns
+// logits [16c, 16c+16) of this thread's row, -FLT_MAX past E (finite, so that its top-k key is
+// not a NaN; warp-collective); release() is called after the last logit read. row: token row in
+// the tile (0..127); lt: index of the tile among those this CTA processes; dll: the row's
+// Gaussian log-likelihood difference (read by group 1); meta: the tile's metadata
+// (load_tile_meta); n_in: completed phases of bar_in (identical in all 256 threads).
+//
+// Softmax in two passes over each group's columns: pass A finds the row maximum and top-k keys
+// (merged across the groups through shared memory); pass B forms e = exp(z - max), its row sum,
+// the bin sums of e and the saved scores (e is saved with 1/sum kept per row, so that nothing
+// waits for the sum before storing). Group 0 then writes the top-k outputs and the permutation's
+// pair counts, group 1 the modality score; both write the per-(tile, sample) partial sums of the
+// joint table (eq. 12), each a half of the values. With the fused permutation, after the CTA's
+// last tile the first warp arrives on es.perm_go once all rows are counted.
 template <int KM, class Src, class Release>
 __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release& release, int tile,
-                              int row, int lt, float dll, const TileMeta& meta, const EpiSmem& es,
-                              const WaitCtx& wc, uint32_t& n_in, bool last_tile) {
+                              int grp, int row, int lt, float dll, const TileMeta& meta,
+                              const EpiSmem& es, const WaitCtx& wc, uint32_t& n_in, bool last_tile) {
   const Dims& dm = p.dm;
   const int E = dm.E, K = dm.K, k = dm.k;
   const int wg = row >> 5, lane = row & 31;
   const int j = tile * kTileRows + row;
   const bool valid = j < dm.T;
   const int nch = (E + 15) >> 4;
+  const int nc0 = epi_split(dm);
+  const bool split = nc0 < nch;
+  const int cb = grp ? nc0 : 0, ce = grp ? nch : nc0;
   const uint32_t imask = (1u << (32 - __clz(max(nch * 16 - 1, 1)))) - 1u;
+  const uint32_t xph = static_cast<uint32_t>(lt & 1);
 
-  // pass A: softmax max and top-k keys, even and odd columns in two independent lists (two
-  // dependency chains), merged at the end
+  // pass A: row maximum and top-k keys of this group's columns, even and odd columns in two
+  // independent lists (two dependency chains), merged at the end
   float tk[KM], tk2[KM];
 #pragma unroll
   for (int i = 0; i < KM; ++i) tk[i] = tk2[i] = -CUDART_INF_F;
   float mx = -CUDART_INF_F, mx2 = -CUDART_INF_F;
 #pragma unroll 1
-  for (int c = 0; c < nch; ++c) {
+  for (int c = cb; c < ce; ++c) {
     float v[16];
     src.load16(c, v);
 #pragma unroll
@@ -337,36 +369,41 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
   mx = fmaxf(mx, mx2);
 #pragma unroll
   for (int i = 0; i < KM; ++i) topk_push<KM>(tk, tk2[i]);
-  // pass B: softmax denominator (four partial sums, added in a fixed order)
-  const float mxl = mx * kLog2e;
-  float sum = 0.f;
-#pragma unroll 1
-  for (int c = 0; c < nch; ++c) {
-    float v[16];
-    src.load16(c, v);
-    float ps[4] = {0.f, 0.f, 0.f, 0.f};
+  es.xmax[grp * 128 + row] = mx;
+  if (grp == 1 && split) {
 #pragma unroll
-    for (int t = 0; t < 16; ++t) ps[t & 3] += exp2f(fmaf(v[t], kLog2e, -mxl));
-    sum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
+    for (int i = 0; i < KM; ++i) es.xtk[i * 128 + row] = tk[i];
   }
-  const float inv = 1.f / sum;
-  if (valid && !(isfinite(mx) && isfinite(sum) && sum > 0.f)) atomicOr(p.ws.status, kStatusData);
-  // pass C: g, saved g, bin probabilities
+  mbar_arrive(es.xbar + 0);
+  if (!mbar_wait(es.xbar + 0, xph, wc)) return;
+  mx = fmaxf(es.xmax[row], es.xmax[128 + row]);
+  if (grp == 0 && split) {
+#pragma unroll
+    for (int i = 0; i < KM; ++i) topk_push<KM>(tk, es.xtk[i * 128 + row]);
+  }
+
+  // pass B: e = exp(z - max), its sum, the bin sums of e and the saved scores
+  const float mxl = mx * kLog2e;
   float* grow = p.ws.gsave + static_cast<size_t>(valid ? j : 0) * E;
   float* prow = es.p_s + row;                       // p_s[b][row] at prow[b * kPsStride]
   const bool vec = (E & 3) == 0;
   const bool stg = es.stg != nullptr;
-  float run = 0.f;
-  int cnt = 0, bin = 0;
-  if (!dm.contig_bins)
+  float sum = 0.f, run = 0.f;
+  int cnt = 0, bin = split && grp ? 16 * nc0 / dm.N_B : 0;
+  if (!dm.contig_bins && grp == 0)
     for (int b = 0; b < K; ++b) prow[b * kPsStride] = 0.f;
-  if (stg && lt > 0 && !mbar_wait(es.stg_free, static_cast<uint32_t>((lt - 1) & 1), wc)) return;
+  if (stg && lt > 0 && !mbar_wait(es.stg_free + grp, static_cast<uint32_t>((lt - 1) & 1), wc)) return;
 #pragma unroll 1
-  for (int c = 0; c < nch; ++c) {
+  for (int c = cb; c < ce; ++c) {
     float v[16];
     src.load16(c, v);
+    float ps[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int t = 0; t < 16; ++t) v[t] = exp2f(fmaf(v[t], kLog2e, -mxl)) * inv;
+    for (int t = 0; t < 16; ++t) {
+      v[t] = exp2f(fmaf(v[t], kLog2e, -mxl));
+      ps[t & 3] += v[t];
+    }
+    sum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
     if (stg) {
       uint8_t* rb = es.stg + (c >> 1) * 16384 + row * 128;
 #pragma unroll
@@ -389,6 +426,7 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
     if (dm.contig_bins) {              // bins are runs of N_B experts, N_B a multiple of 4
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
+        if (c * 16 + 4 * q >= E) break;   // padding columns (e = 0 past E) end the last bin
         run += (v[4 * q] + v[4 * q + 1]) + (v[4 * q + 2] + v[4 * q + 3]);
         cnt += 4;
         if (cnt == dm.N_B) {
@@ -398,107 +436,127 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
           ++bin;
         }
       }
-    } else {                           // any expert -> bin map
+    } else {                           // any expert -> bin map (group 0 holds every column)
 #pragma unroll
       for (int t = 0; t < 16; ++t)
         if (c * 16 + t < E) prow[__ldg(p.ws.expert_bin + c * 16 + t) * kPsStride] += v[t];
     }
   }
   release();
-  if (stg) {                       // one thread stores the staged scores (rows >= T are clipped)
+  if (stg) {                      // the group's first thread stores its staged blocks (rows >= T clipped)
     fence_proxy_async_smem();
-    mbar_arrive(es.stg_full);
-    if (row == 0 && mbar_wait(es.stg_full, static_cast<uint32_t>(lt & 1), wc)) {
-      for (int b = 0; b * 32 < E; ++b) tma_store_2d(es.tmG, es.stg + b * 16384, 32 * b, tile * kTileRows);
+    mbar_arrive(es.stg_full + grp);
+    if (row == 0 && mbar_wait(es.stg_full + grp, static_cast<uint32_t>(lt & 1), wc)) {
+      for (int b = cb >> 1; cb < ce && b < (ce + 1) >> 1; ++b)
+        tma_store_2d(es.tmG, es.stg + b * 16384, 32 * b, tile * kTileRows);
       tma_store_commit();
     }
   }
+  es.xsum[grp * 128 + row] = sum;
+  mbar_arrive(es.xbar + 1);
+  if (!mbar_wait(es.xbar + 1, xph, wc)) return;
+  const float tot = es.xsum[row] + es.xsum[128 + row];
+  const float inv = 1.f / tot;
+  // this group's bins (all of them for group 0 without a split): e sums -> probabilities
+  const int kb0 = split && grp ? 16 * nc0 / dm.N_B : 0;
+  const int kb1 = split && !grp ? 16 * nc0 / dm.N_B : (grp && !split ? 0 : K);
+  for (int b = kb0; b < kb1; ++b) prow[b * kPsStride] = valid ? prow[b * kPsStride] * inv : 0.f;
 
-  // modality score of this token (eq. 9 for two modalities, or the provided scores)
   float Mv = 0.f, Mt = 0.f, dv = 0.f, dt = 0.f;
-  if (valid) {
-    if (p.M_in) {
-      const float2 m = __ldg(reinterpret_cast<const float2*>(p.M_in) + j);
-      Mv = m.x;
-      Mt = m.y;
-      dv = Mv - 0.5f;
-      dt = Mt - 0.5f;
-    } else {
-      const float y = dll * p.inv_tau;
-      Mv = sigmoid_acc(y);
-      Mt = sigmoid_acc(-y);
-      dv = 0.5f * tanhf(0.5f * y);
-      dt = -dv;
-      if (p.M_out) reinterpret_cast<float2*>(p.M_out)[j] = make_float2(Mv, Mt);
-    }
-    // top-k outputs: indices from the keys; weights = the staged scores, or recomputed from the
-    // keys' logits when the scores are not staged
-    float w[KM];
-    float wsum = 0.f;
-#pragma unroll
-    for (int i = 0; i < KM; ++i) {
-      w[i] = 0.f;
-      if (i < k) {
-        if (stg) {
-          const uint32_t e = static_cast<uint32_t>(topk_index(tk[i], imask));
-          const uint32_t qd = ((e & 31u) >> 2) ^ static_cast<uint32_t>(row & 7);
-          w[i] = *reinterpret_cast<const float*>(es.stg + (e >> 5) * 16384u + row * 128 + (qd << 4) + (e & 3u) * 4u);
-        } else {
-          w[i] = exp2f(fmaf(topk_logit(tk[i], imask), kLog2e, -mxl)) * inv;
-        }
-      }
-      wsum += w[i];
-    }
-    const float wsc = dm.renorm ? 1.f / wsum : 1.f;
-    int32_t* ti = p.topk_idx + static_cast<size_t>(j) * k;
-    float* tw = p.topk_w + static_cast<size_t>(j) * k;
-#pragma unroll
-    for (int i = 0; i < KM; ++i) {
-      if (i < k) {
-        ti[i] = topk_index(tk[i], imask);
-        tw[i] = w[i] * wsc;
-      }
-    }
-    if (p.bin_prob)
-      for (int kb = 0; kb < K; ++kb) p.bin_prob[static_cast<size_t>(j) * K + kb] = prow[kb * kPsStride];
-  } else {
-    for (int b = 0; b < K; ++b) prow[b * kPsStride] = 0.f;
-  }
-  if (p.perm.perm_token) {           // (token, bin) pairs of this warp's rows, per bin
-    uint32_t bins = 0u;
+  if (grp == 0) {
+    if (valid && !(isfinite(mx) && isfinite(tot) && tot > 0.f)) atomicOr(p.ws.status, kStatusData);
+    // top-k outputs: indices from the keys; weights = the staged e, or e recomputed from the
+    // keys' logits when the scores are not staged, times 1/sum
     if (valid) {
+      float w[KM];
+      float wsum = 0.f;
+#pragma unroll
+      for (int i = 0; i < KM; ++i) {
+        w[i] = 0.f;
+        if (i < k) {
+          if (stg) {
+            const uint32_t e = static_cast<uint32_t>(topk_index(tk[i], imask));
+            const uint32_t qd = ((e & 31u) >> 2) ^ static_cast<uint32_t>(row & 7);
+            w[i] = *reinterpret_cast<const float*>(es.stg + (e >> 5) * 16384u + row * 128 + (qd << 4) + (e & 3u) * 4u) * inv;
+          } else {
+            w[i] = exp2f(fmaf(topk_logit(tk[i], imask), kLog2e, -mxl)) * inv;
+          }
+        }
+        wsum += w[i];
+      }
+      const float wsc = dm.renorm ? 1.f / wsum : 1.f;
+      int32_t* ti = p.topk_idx + static_cast<size_t>(j) * k;
+      float* tw = p.topk_w + static_cast<size_t>(j) * k;
 #pragma unroll
       for (int i = 0; i < KM; ++i) {
         if (i < k) {
-          const int e = topk_index(tk[i], imask);
-          bins |= 1u << (dm.contig_bins ? e / dm.N_B : __ldg(p.ws.expert_bin + e));
+          ti[i] = topk_index(tk[i], imask);
+          tw[i] = w[i] * wsc;
         }
       }
     }
-    for (int kb = 0; kb < K; ++kb) {
-      const int c = __popc(__ballot_sync(0xffffffffu, (bins >> kb) & 1u));
-      if (lane == kb && c) atomicAdd(es.ctot + kb, c);
+    if (p.perm.perm_token) {         // (token, bin) pairs of this warp's rows, per bin
+      uint32_t bins = 0u;
+      if (valid) {
+#pragma unroll
+        for (int i = 0; i < KM; ++i) {
+          if (i < k) {
+            const int e = topk_index(tk[i], imask);
+            bins |= 1u << (dm.contig_bins ? e / dm.N_B : __ldg(p.ws.expert_bin + e));
+          }
+        }
+      }
+      for (int kb = 0; kb < K; ++kb) {
+        const int c = __popc(__ballot_sync(0xffffffffu, (bins >> kb) & 1u));
+        if (lane == kb && c) atomicAdd(es.ctot + kb, c);
+      }
     }
+  } else {
+    // modality score of this token (eq. 9 for two modalities, or the provided scores)
+    if (valid) {
+      if (p.M_in) {
+        const float2 m = __ldg(reinterpret_cast<const float2*>(p.M_in) + j);
+        Mv = m.x;
+        Mt = m.y;
+        dv = Mv - 0.5f;
+        dt = Mt - 0.5f;
+      } else {
+        const float y = dll * p.inv_tau;
+        Mv = sigmoid_acc(y);
+        Mt = sigmoid_acc(-y);
+        dv = 0.5f * tanhf(0.5f * y);
+        dt = -dv;
+        if (p.M_out) reinterpret_cast<float2*>(p.M_out)[j] = make_float2(Mv, Mt);
+      }
+      p.ws.ginv[j] = inv;
+    }
+    float* mrow = es.m_s + row;
+    mrow[0] = dv;
+    mrow[kPsStride] = dt;
+    mrow[2 * kPsStride] = Mv;
+    mrow[3 * kPsStride] = Mt;
+    mrow[4 * kPsStride] = 1.f;
   }
-  float* mrow = es.m_s + row;
-  mrow[0] = dv;
-  mrow[kPsStride] = dt;
-  mrow[2 * kPsStride] = Mv;
-  mrow[3 * kPsStride] = Mt;
-  mrow[4 * kPsStride] = 1.f;
-  __syncwarp();
+  mbar_arrive(es.xbar + 2);
+  if (!mbar_wait(es.xbar + 2, xph, wc)) return;
+  if (valid && p.bin_prob)
+    for (int b = grp; b < K; b += 2) p.bin_prob[static_cast<size_t>(j) * K + b] = prow[b * kPsStride];
 
-  // partial sums of the joint table: one piece per (tile, sample); each warp sums its 32 rows
-  // (lane = value), the four warp partials are then added in warp order. The rows of a sample
-  // are contiguous: a ballot over the rows' sample ids gives the warp's range.
+  // partial sums of the joint table: one piece per (tile, sample); group g sums the values of
+  // its half over the rows of each lane quarter (lane = value), the four quarters' partials are
+  // then added in quarter order. The rows of a sample are contiguous: a ballot over the rows'
+  // sample ids gives the warp's range.
   const int NV = piece_values(K);
+  const int NVh = (NV + 1) >> 1;
+  const int vb = grp ? NVh : 0, ve = grp ? NV : NVh;
+  const int tid = grp * 128 + row;
   const int s0 = meta.s0, s1 = meta.s1;
   for (int s = s0; s <= s1; ++s) {
     const uint32_t mine = __ballot_sync(0xffffffffu, meta.row_sample == s);
     const int r0 = 32 * wg + (mine ? __ffs(mine) - 1 : 0);
     const int r1 = 32 * wg + (mine ? 32 - __clz(mine) : 0);
     float* wp = es.wpart + ((n_in & 1) * 4 + wg) * kMaxNV;
-    for (int v = lane; v < NV; v += 32) {
+    for (int v = vb + lane; v < ve; v += 32) {
       // value v: kind v / K over bin v % K (kind 0: Q, 1..4: weighted by m_s rows 0..3),
       // or, past 5K, the plain sum of m_s row v - 5K
       const int kind = v < 5 * K ? v / K : 0;
@@ -514,16 +572,16 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
     const float* w0 = es.wpart + (n_in & 1) * 4 * kMaxNV;
     ++n_in;
     float* piece = p.ws.pieces + static_cast<size_t>(meta.pbase + (s - s0)) * dm.pstride;
-    for (int v = row; v < NV; v += 128)
+    for (int v = tid; v < NV; v += 256)
       piece[v] = ((w0[v] + w0[kMaxNV + v]) + w0[2 * kMaxNV + v]) + w0[3 * kMaxNV + v];
   }
   if (stg && row == 0) {            // the staging may be rewritten once the store has read it
     tma_store_wait_read<0>();
-    mbar_arrive(es.stg_free);
+    mbar_arrive(es.stg_free + grp);
   }
   __threadfence();
   mbar_arrive(es.bar_out);
-  if (wg == 0) {                        // the first warp announces the pieces, reduces samples
+  if (grp == 0 && wg == 0) {            // the first warp announces the pieces, reduces samples
     bool ok = true;
     if (lane == 0) ok = mbar_wait(es.bar_out, static_cast<uint32_t>(lt & 1), wc);
     ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -541,7 +599,7 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
       if (last) {
         __threadfence();
         const bool known = s == s0 || s == s1;
-        sample_reduce(p, s, es.red, known ? pb : -1, pe, nt);
+        sample_reduce(p, s, es.red, known ? pb : -1, pe, nt, false);
       }
     }
   }
@@ -735,14 +793,18 @@ __host__ __device__ inline size_t fwd_smem_bytes(int N, int n_stages, int d, int
   if (stg) b += fwd_stg_bytes(E);
   if (gauss) b += 2u * sizeof(float) * static_cast<size_t>(round_up(d, kFwdBK));
   b += sizeof(float) * (epi_smem_floats(K) + 256u + 8u);
-  b += sizeof(uint64_t) * (2u * n_stages + 17u + kCoefBars);
+  b += sizeof(uint64_t) * (2u * n_stages + 19u + kEpiBars + kCoefBars);
   b += 16u;
   return b + 1024u;   // alignment slack
 }
 
-// 10 warps: three share a sub-partition's 16K registers, so a thread gets at most 168.
+// Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-5 epilogue group 0, then (Gaussian
+// score) warps 6-9 Gaussian and 10-13 epilogue group 1, or (provided scores) warps 6-9 epilogue
+// group 1. With 14 warps four share a sub-partition's 16K registers: 128 per thread.
+constexpr int fwd_threads(bool gauss) { return gauss ? 448 : 320; }
+
 template <bool kGauss, int KM>
-__global__ void __launch_bounds__(kGauss ? 320 : 192, 1)
+__global__ void __launch_bounds__(fwd_threads(kGauss), 1)
 k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
                 const __grid_constant__ CUtensorMap tmG, const FwdParams p, const int N,
                 const int n_stages, const int use_stg) {
@@ -775,14 +837,13 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   uint64_t* g_full = reinterpret_cast<uint64_t*>(q);    q += 16;
   uint64_t* g_empty = reinterpret_cast<uint64_t*>(q);   q += 16;
   uint64_t* drain = reinterpret_cast<uint64_t*>(q);     q += 8;
-  uint64_t* bar_in = reinterpret_cast<uint64_t*>(q);    q += 8;
-  uint64_t* bar_out = reinterpret_cast<uint64_t*>(q);   q += 8;
+  uint64_t* ebars = reinterpret_cast<uint64_t*>(q);     q += 8 * kEpiBars;
   uint64_t* coef_bar = reinterpret_cast<uint64_t*>(q);  q += 8 * kCoefBars;
   uint64_t* coef_issued = reinterpret_cast<uint64_t*>(q);  q += 8;
   uint64_t* gc_bar = reinterpret_cast<uint64_t*>(q);    q += 8;
   uint64_t* perm_go = reinterpret_cast<uint64_t*>(q);   q += 8;
-  uint64_t* stg_full = reinterpret_cast<uint64_t*>(q);  q += 8;
-  uint64_t* stg_free = reinterpret_cast<uint64_t*>(q);  q += 8;
+  uint64_t* stg_full = reinterpret_cast<uint64_t*>(q);  q += 16;
+  uint64_t* stg_free = reinterpret_cast<uint64_t*>(q);  q += 16;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q); q += 4;
   int* abort_flag = reinterpret_cast<int*>(q);
 
@@ -797,22 +858,21 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(acc_full + i, 1);
-      mbar_init(acc_empty + i, 128);
+      mbar_init(acc_empty + i, 256);             // both epilogue groups read the accumulator
       mbar_init(g_full + i, 128);
       mbar_init(g_empty + i, 128);
+      mbar_init(stg_full + i, 128);
+      mbar_init(stg_free + i, 1);
     }
     mbar_init(drain, 1);
-    mbar_init(bar_in, 128);
-    mbar_init(bar_out, 128);
+    init_epi_bars(ebars);
     mbar_init(coef_bar, 256);
     for (int i = 1; i < kCoefBars; ++i) mbar_init(coef_bar + i, 128);
     mbar_init(coef_issued, 256);
     mbar_init(gc_bar, 256);
     mbar_init(perm_go, 1);
-    int* ctot = epi_smem(epi, dm.K, bar_in, bar_out).ctot;
+    int* ctot = epi_smem(epi, dm.K, ebars).ctot;
     for (int i = 0; i < kMaxBins; ++i) ctot[i] = 0;
-    mbar_init(stg_full, 128);
-    mbar_init(stg_free, 1);
     fence_mbar_init();
     tma_prefetch_desc(&tmX);
     tma_prefetch_desc(&tmW);
@@ -828,7 +888,7 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   pdl_wait();
   pdl_trigger();
 
-  if (kGauss && warp >= 2) {
+  if (kGauss && warp >= 2 && warp < 10) {
     // this CTA's Gaussian coefficients (eqs. 8-9), float4 {ga[2i], ga[2i+1], gb[2i], gb[2i+1]}
     // per feature pair i, computed in the order in which the CTA walks the K-blocks, in chunks
     // of eight blocks (256 pairs): chunk 0 by the epilogue and Gaussian warps together, one pair
@@ -958,11 +1018,12 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       wd.abort_flag = &dummy;
       mbar_wait(drain, 0, wd);
     }
-  } else if (warp < 6) {
-    // ---------------------------------------------------------------- epilogue (4 warps)
+  } else if (warp < 6 || warp >= (kGauss ? 10 : 6)) {
+    // ---------------------------------------------------------------- epilogue (2 x 4 warps)
+    const int grp = warp < 6 ? 0 : 1;        // column half of the logits
     const int lg = warp & 3;                 // TMEM lane group accessible to this warp
     const int row = lg * 32 + lane;          // tile row == TMEM lane == token offset
-    EpiSmem es = epi_smem(epi, dm.K, bar_in, bar_out);
+    EpiSmem es = epi_smem(epi, dm.K, ebars);
     es.perm_go = perm_go;
     if (use_stg) {
       es.stg = stg;
@@ -988,10 +1049,12 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     };
     const uint32_t tl = tmem_base + (static_cast<uint32_t>(lg * 32) << 16);
     float gc = 0.f;                          // constant term of eq. (8), -1/2 sum of the parts
-    if (kGauss && mbar_wait(gc_bar, 0, wc)) {
+    if (kGauss && grp == 1 && mbar_wait(gc_bar, 0, wc)) {
       for (int w = 0; w < 8; ++w) gc += gred[w];
       gc *= -0.5f;
     }
+    // the sample reduction's code into the instruction cache while the first tile streams in
+    if (grp == 0 && lg == 0) sample_reduce(p, 0, es.red, 0, 1, 1, true);
     uint32_t n_in = 0;
     int lt = 0;
     for (int tile = t_beg; tile < t_end; ++tile, ++lt) {
@@ -1001,13 +1064,13 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       if (!mbar_wait(acc_full + buf, use & 1u, wc)) break;
       tc_fence_after();
       float dll = 0.f;
-      if (kGauss) {
+      if (kGauss && grp == 1) {
         if (!mbar_wait(g_full + buf, use & 1u, wc)) break;
         dll = dll_s[buf * 128 + row] + gc;
         mbar_arrive(g_empty + buf);
       }
       epilogue_tile<KM>(p, Src{tl + static_cast<uint32_t>(buf * N), dm.E}, Rel{acc_empty + buf},
-                        tile, row, lt, dll, meta, es, wc, n_in, tile == t_end - 1);
+                        tile, grp, row, lt, dll, meta, es, wc, n_in, tile == t_end - 1);
     }
     if (use_stg && row == 0) tma_store_wait_all<0>();   // the score stores complete before exit
   } else {
@@ -1016,7 +1079,7 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     // per stage a lane reads one float4 of coefficients and one 4-byte word of each of its
     // warp's rows, and keeps one running sum per row; a butterfly over the lanes gives the row
     // totals at the end of the tile.
-    if (kGauss) {
+    if (kGauss) {                            // (warps 6-9)
       const int gw = warp - 6;
       const int gt = gw * 32 + lane;
       bool ok = true;
@@ -1061,8 +1124,9 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   // once their part of the CTA's tiles is done; the stage buffers are free after perm_go
   if (p.perm.perm_token) {
     int* ps = reinterpret_cast<int*>(stage);
-    const int* ctot = epi_smem(epi, dm.K, bar_in, bar_out).ctot;
-    if (kGauss && warp >= 6) perm_tail<KM>(p, t_beg, t_end, threadIdx.x - 192, 4, 1, ctot, ps, perm_go, wc);
+    const int* ctot = epi_smem(epi, dm.K, ebars).ctot;
+    if (kGauss && warp >= 6 && warp < 10)
+      perm_tail<KM>(p, t_beg, t_end, threadIdx.x - 192, 4, 1, ctot, ps, perm_go, wc);
     if (!kGauss && warp < 2) perm_tail<KM>(p, t_beg, t_end, threadIdx.x, 2, 1, ctot, ps, perm_go, wc);
   }
 
@@ -1074,8 +1138,8 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
 
 // ------------------------------------------------------------------ FFMA forward (fp32)
 // 128 tokens per block, 512 threads: thread (row r = t/4, quarter q = t%4) accumulates the
-// logits of experts e = q + 4i over d and a quarter of the Gaussian sum; threads 0..127 then
-// run the same epilogue as the tensor-core path (logits read from shared memory).
+// logits of experts e = q + 4i over d and a quarter of the Gaussian sum; threads 0..255 then
+// run the same two-group epilogue as the tensor-core path (logits read from shared memory).
 constexpr int kF32MaxE = 64;
 
 __host__ __device__ inline size_t f32_smem_floats(const Dims& dm) {
@@ -1101,8 +1165,8 @@ k_router_fwd_f32(const FwdParams p) {
   float* epi = gb + dpad;                  // epilogue tables
   float* dll_s = epi + epi_smem_floats(dm.K);   // [128]
   uint64_t* bars = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(dll_s + 128) + 7) & ~uintptr_t(7));   // [2]
-  int* abort_flag = reinterpret_cast<int*>(bars + 2);
+      (reinterpret_cast<uintptr_t>(dll_s + 128) + 7) & ~uintptr_t(7));   // [kEpiBars]
+  int* abort_flag = reinterpret_cast<int*>(bars + kEpiBars);
 
   const int t = threadIdx.x, r = t >> 2, qd = t & 3;
   const int tile = blockIdx.x;
@@ -1111,8 +1175,7 @@ k_router_fwd_f32(const FwdParams p) {
   pdl_trigger();
   if (t == 0) {
     *abort_flag = 0;
-    mbar_init(bars + 0, 128);
-    mbar_init(bars + 1, 128);
+    init_epi_bars(bars);
     fence_mbar_init();
   }
   float gc = 0.f;
@@ -1161,7 +1224,8 @@ k_router_fwd_f32(const FwdParams p) {
   gacc += __shfl_xor_sync(0xffffffffu, gacc, 2);
   if (qd == 0) dll_s[r] = gacc + gc;
   __syncthreads();
-  if (t < 128) {
+  if (t < 256) {
+    const int grp = t >> 7, row = t & 127;
     struct Src {
       const float* z;
       int E;
@@ -1169,15 +1233,15 @@ k_router_fwd_f32(const FwdParams p) {
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = (16 * c + i < E) ? z[16 * c + i] : -FLT_MAX;
       }
-    } src{zs + t * (E16 + 1), E};
+    } src{zs + row * (E16 + 1), E};
     struct Rel {
       __device__ void operator()() const {}
     } rel;
     WaitCtx wc{abort_flag, p.ws.status, p.limit_ns};
-    const EpiSmem es = epi_smem(epi, dm.K, bars + 0, bars + 1);
+    const EpiSmem es = epi_smem(epi, dm.K, bars);
     uint32_t n_in = 0;
-    const TileMeta meta = load_tile_meta(p, tile, t);   // (no fused permutation on this path)
-    epilogue_tile<KM>(p, src, rel, tile, t, 0, kGauss ? dll_s[t] : 0.f, meta, es, wc, n_in, true);
+    const TileMeta meta = load_tile_meta(p, tile, row);   // (no fused permutation on this path)
+    epilogue_tile<KM>(p, src, rel, tile, grp, row, 0, kGauss ? dll_s[row] : 0.f, meta, es, wc, n_in, true);
   }
 }
 
@@ -1219,12 +1283,12 @@ cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     if (!p.perm.perm_token)
-      return launch_pdl(k, dim3(grid), dim3(gauss ? 320 : 192), smem, s, tmX, tmW, tg, p, N, n_stages,
+      return launch_pdl(k, dim3(grid), dim3(fwd_threads(gauss)), smem, s, tmX, tmW, tg, p, N, n_stages,
                         use_stg ? 1 : 0);
     // the fused permutation has a grid barrier: every CTA must be resident (cooperative launch)
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(gauss ? 320 : 192);
+    cfg.blockDim = dim3(fwd_threads(gauss));
     cfg.dynamicSmemBytes = smem;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
@@ -1240,7 +1304,7 @@ cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
 
 cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s) {
   if (p.dm.E > kF32MaxE) return cudaErrorInvalidValue;
-  const size_t smem = sizeof(float) * f32_smem_floats(p.dm) + sizeof(int) * round_up(p.dm.E, 4) + 64;
+  const size_t smem = sizeof(float) * f32_smem_floats(p.dm) + sizeof(uint64_t) * kEpiBars + 64;
   if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
   const bool gauss = p.M_in == nullptr;
   return dispatch_km(p.dm.k, [&](auto km) -> cudaError_t {

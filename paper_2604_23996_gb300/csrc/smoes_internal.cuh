@@ -41,7 +41,8 @@ struct WsView {
   float* pieces;             // [n_pieces * piece_stride]
   float* mi32;               // [B] per-sample MI for the loss
   float* tabs;               // [B * 3 * K]: a_k, b_k, h_k per sample (backward coefficients)
-  float* gsave;              // [T * E] softmax scores saved by the forward
+  float* gsave;              // [T * E] exp(z_je - max_e z_je) saved by the forward
+  float* ginv;               // [T] 1 / sum_e exp(z_je - max_e z_je): g_je = gsave * ginv
   float* dw_part;            // [G * E * d] per-token-group partial dW
   uint8_t* dz_img;           // [ceil(T/64)][hi|lo][E_pad/64][64 rows][128 B] dz in the MMA layout
   int32_t* perm_scratch;     // permutation block counts [n_blocks * K]
