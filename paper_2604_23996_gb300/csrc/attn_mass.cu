@@ -7,12 +7,15 @@
 //
 // A work item is (sequence, head, pair of adjacent 128-query tiles). The two tiles share one
 // stream of 128-key blocks: for each block the tensor cores form S = Q K^T of both tiles
-// (tcgen05, TMA-fed, accumulators in TMEM, two buffers per tile). Two softmax groups of four
-// warps (one query row per thread, one group per tile) keep the online max, the normaliser
-// l = sum e^(s - max) and the vision mass a = sum e^(s - max) m_j'. The head's score a / l goes
-// to the workspace; the last head of each (sequence, query tile) to finish averages the heads in
-// fixed order and writes M (optionally blended with the carried score by eq. 4). Items are
-// handed out longest first so that the CTAs finish together.
+// (tcgen05, TMA-fed, accumulators in TMEM, two buffers per tile). Four softmax groups of four
+// warps (one query row per thread; a group per tile and half of the 128 keys of a block) keep
+// the online max, the normaliser l = sum e^(s - max) and the vision mass a = sum e^(s - max) m_j'
+// of their keys; at the end of an item the second half's state is merged into the first's (fixed
+// order). Sixteen softmax warps keep the special-function unit, which evaluates one
+// exponential per score, busier than eight could. The head's score a / l goes to the workspace;
+// the last head of each (sequence, query tile) to finish averages the heads in fixed order and
+// writes M (optionally blended with the carried score by eq. 4). Items are handed out longest
+// first so that the CTAs finish together.
 #include <cuda_bf16.h>
 #include <math_constants.h>
 
@@ -27,8 +30,11 @@ constexpr int kAT = 128;                      // queries per tile, keys per bloc
 constexpr int kHd = 128;                      // head dimension handled here
 constexpr uint32_t kTile = kAT * kHd * 2;     // bytes of one Q tile or K block (2 swizzle atoms)
 
+constexpr int kHalf = kAT / 2;                // keys of a block per softmax group
+constexpr int kAttnThreads = 64 + 4 * 128;    // producer, MMA issuer, four softmax groups
+
 struct AttnLayout {
-  uint32_t q, k, mk, bars, total;
+  uint32_t q, k, mk, mrg, bars, total;
 };
 
 __host__ __device__ inline AttnLayout attn_layout(int n_ks) {
@@ -36,8 +42,9 @@ __host__ __device__ inline AttnLayout attn_layout(int n_ks) {
   uint32_t o = 0;
   L.q = o;    o += 2u * kTile;                             // two Q tiles [2 atoms][128 rows][128 B]
   L.k = o;    o += static_cast<uint32_t>(n_ks) * kTile;    // K blocks
-  L.mk = o;   o += 2u * 2u * 2u * kAT * 4u;                // bias*log2e [128] | m [128]: group x buffer
-  L.bars = o; o += 8u * (2u * n_ks + 24u) + 32u;
+  L.mk = o;   o += 4u * 2u * 2u * kHalf * 4u;              // bias*log2e [64] | m [64]: group x buffer
+  L.mrg = o;  o += 2u * 2u * 3u * kAT * 4u;                // second half's (max, l, a): tile x buffer
+  L.bars = o; o += 8u * (2u * n_ks + 30u) + 32u;
   L.total = o + 1024u;
   return L;
 }
@@ -93,7 +100,7 @@ __device__ __forceinline__ int kblocks_of(const AttnParams& p, int qt) {
 }
 
 template <bool kFloatM>
-__global__ void __launch_bounds__(320, 1)
+__global__ void __launch_bounds__(kAttnThreads, 1)
 k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
             const AttnParams p, const int n_ks) {
   extern __shared__ uint8_t smem_raw[];
@@ -102,6 +109,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   uint8_t* qs = base + L.q;
   uint8_t* ks = base + L.k;
   float* mk = reinterpret_cast<float*>(base + L.mk);
+  float* mrg = reinterpret_cast<float*>(base + L.mrg);
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
   uint64_t* kfull = bars;
   uint64_t* kempty = bars + n_ks;
@@ -109,11 +117,12 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   uint64_t* q_empty = q_full + 2;       // [2]
   uint64_t* s_full = q_full + 4;        // [tile][buf]
   uint64_t* s_empty = q_full + 8;       // [tile][buf]
-  uint64_t* mk_bar = q_full + 12;       // [tile][buf] keys' (bias, m) staged by that group
-  uint64_t* out_bar = q_full + 16;      // [tile] head results of the tile written
-  uint64_t* dec_bar = q_full + 18;      // [tile] the ticket decision of the tile is published
-  uint64_t* drain = q_full + 20;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 22);
+  uint64_t* mk_bar = q_full + 12;       // [group][buf] keys' (bias, m) staged by that group
+  uint64_t* out_bar = q_full + 20;      // [tile] head results of the tile written
+  uint64_t* dec_bar = q_full + 22;      // [tile] the ticket decision of the tile is published
+  uint64_t* mrg_bar = q_full + 24;      // [tile] the second half's state of the item is written
+  uint64_t* drain = q_full + 26;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 28);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
   volatile uint32_t* decision = reinterpret_cast<volatile uint32_t*>(tmem_slot + 2);   // [2]
 
@@ -132,12 +141,13 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       mbar_init(q_empty + t, 1);
       mbar_init(out_bar + t, 128);
       mbar_init(dec_bar + t, 1);
+      mbar_init(mrg_bar + t, 128);
       for (int i = 0; i < 2; ++i) {
         mbar_init(s_full + 2 * t + i, 1);
-        mbar_init(s_empty + 2 * t + i, 128);
-        mbar_init(mk_bar + 2 * t + i, 128);
+        mbar_init(s_empty + 2 * t + i, 256);     // both key halves read the scores
       }
     }
+    for (int i = 0; i < 8; ++i) mbar_init(mk_bar + i, 128);
     mbar_init(drain, 1);
     fence_mbar_init();
     tma_prefetch_desc(&tmQ);
@@ -243,15 +253,18 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       mbar_wait(drain, 0, wd);
     }
   } else {
-    // ---------------------------------------------------------------- softmax groups (2 x 4 warps)
-    const int t = (warp - 2) >> 2;             // query tile of the pair handled by this group
+    // ---------------------------------------------------------------- softmax groups (4 x 4 warps)
+    const int grp = (warp - 2) >> 2;
+    const int t = grp & 1;                     // query tile of the pair handled by this group
+    const int hf = grp >> 1;                   // half of each key block: keys [64 hf, 64 hf + 64)
     const int lg = warp & 3;
     const int row = lg * 32 + lane;            // query row in the tile == TMEM lane
-    const int gt = threadIdx.x - 64 - 128 * t; // 0..127 inside the group
-    float* mkg = mk + 2 * t * 2 * kAT;         // this group's staging: [buf][bias 128 | m 128]
+    const int gt = threadIdx.x - 64 - 128 * grp; // 0..127 inside the group
+    float* mkg = mk + grp * 2 * kAT;           // this group's staging: [buf][bias 64 | m 64]
+    float* mrt = mrg + t * 2 * 3 * kAT;        // the tile's merge buffers: [item parity][3][128]
     uint64_t* sfull = s_full + 2 * t;
     uint64_t* sempty = s_empty + 2 * t;
-    uint64_t* mkbar = mk_bar + 2 * t;
+    uint64_t* mkbar = mk_bar + 2 * grp;
     int blk = 0;
     int ng = 0;                                // items this group has processed
     for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
@@ -263,13 +276,13 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       float mrun = -CUDART_INF_F;
       float l4[4] = {0.f, 0.f, 0.f, 0.f}, a4[4] = {0.f, 0.f, 0.f, 0.f};
       bool ok = true;
-      // keys' (bias * log2 e, carried score) of block kb for thread gt, masked keys get -inf;
-      // loaded one block ahead so that the global round trip overlaps the current block
+      // keys' (bias * log2 e, carried score) of this half of block kb for thread gt < 64, masked
+      // keys get -inf; loaded one block ahead so that the global round trip overlaps the block
       auto key_vals = [&](int kb, float& bias, float& m) {
-        const int key = kb * kAT + gt;
+        const int key = kb * kAT + kHalf * hf + gt;
         bias = -CUDART_INF_F;
         m = 0.f;
-        if (key < p.S) {
+        if (gt < kHalf && key < p.S) {
           const size_t tk = static_cast<size_t>(w.b) * p.S + key;
           bias = p.key_bias ? __ldg(p.key_bias + tk) * 1.4426950408889634f : 0.f;
           m = kFloatM ? __ldg(p.m_prev + tk) : static_cast<float>(__ldg(p.is_vision + tk) != 0);
@@ -280,25 +293,28 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       for (int kb = 0; kb < nkb; ++kb, ++blk) {
         const int buf = blk & 1;
         const uint32_t use = static_cast<uint32_t>(blk >> 1);
-        mkg[buf * 2 * kAT + gt] = nb_bias;
-        mkg[buf * 2 * kAT + kAT + gt] = nb_m;
+        if (gt < kHalf) {
+          mkg[buf * kAT + gt] = nb_bias;
+          mkg[buf * kAT + kHalf + gt] = nb_m;
+        }
         mbar_arrive(mkbar + buf);
         if (kb + 1 < nkb) key_vals(kb + 1, nb_bias, nb_m);
         if (!mbar_wait(mkbar + buf, use & 1u, wc)) { ok = false; break; }
         if (!mbar_wait(sfull + buf, use & 1u, wc)) { ok = false; break; }
         tc_fence_after();
         const uint32_t ta = tmem + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>((2 * t + buf) * kAT);
-        const float4* bias4 = reinterpret_cast<const float4*>(mkg + buf * 2 * kAT);
-        const float4* m4 = reinterpret_cast<const float4*>(mkg + buf * 2 * kAT + kAT);
+        const float4* bias4 = reinterpret_cast<const float4*>(mkg + buf * kAT);
+        const float4* m4 = reinterpret_cast<const float4*>(mkg + buf * kAT + kHalf);
         const bool diag = p.causal && kb == qt;
 #pragma unroll 1
-        for (int c = 0; c < kAT / 32; ++c) {
+        for (int cc = 0; cc < kHalf / 32; ++cc) {
+          const int c = 2 * hf + cc;            // 32-key chunk of the block
           float v[32];
           tmem_ld32(ta + 32u * c, v);
           float cm[4] = {-CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F, -CUDART_INF_F};
 #pragma unroll
           for (int i4 = 0; i4 < 8; ++i4) {
-            const float4 bb = bias4[c * 8 + i4];
+            const float4 bb = bias4[cc * 8 + i4];
             const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
             const int i = 4 * i4;
             fma2(v[i], v[i + 1], v[i], v[i + 1], p.scale_log2, p.scale_log2, bv[0], bv[1]);
@@ -324,7 +340,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
             }
 #pragma unroll
             for (int i4 = 0; i4 < 8; ++i4) {
-              const float4 mm = m4[c * 8 + i4];
+              const float4 mm = m4[cc * 8 + i4];
               const float mv[4] = {mm.x, mm.y, mm.z, mm.w};
               const int i = 4 * i4;
               float t0, t1, t2, t3;
@@ -342,14 +358,36 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         mbar_arrive(sempty + buf);
       }
       if (!ok) break;
-      const float l = (l4[0] + l4[1]) + (l4[2] + l4[3]);
-      const float a = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+      float l = (l4[0] + l4[1]) + (l4[2] + l4[3]);
+      float a = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+      const uint32_t nt = static_cast<uint32_t>(ng++);   // this item's phase of the group's barriers
+      // the second half hands its state to the first, which merges it (maxima in log2 units)
+      float* mb = mrt + (nt & 1u) * 3 * kAT;
+      if (hf == 1) {
+        mb[row] = mrun;
+        mb[kAT + row] = l;
+        mb[2 * kAT + row] = a;
+        mbar_arrive(mrg_bar + t);
+        continue;
+      }
+      if (!mbar_wait(mrg_bar + t, nt & 1u, wc)) break;
+      {
+        const float m1 = mb[row], l1 = mb[kAT + row], a1 = mb[2 * kAT + row];
+        const float mm = fmaxf(mrun, m1);
+        if (mm == -CUDART_INF_F) {
+          l = 0.f;
+          a = 0.f;
+        } else {
+          const float c0 = ex2(mrun - mm), c1 = ex2(m1 - mm);
+          l = l * c0 + l1 * c1;
+          a = a * c0 + a1 * c1;
+        }
+      }
       // head result, then the head average of the tile by the last head to finish
       const bool valid = q < p.S;
       const size_t tok = static_cast<size_t>(w.b) * p.S + q;
       if (valid) p.part[static_cast<size_t>(w.h) * p.T + tok] = a / l;
       __threadfence();
-      const uint32_t nt = static_cast<uint32_t>(ng++);   // this item's phase of the group's barriers
       mbar_arrive(out_bar + t);
       if (gt == 0) {
         uint32_t last = 0u;
@@ -396,7 +434,7 @@ cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const 
   auto k = p.m_prev ? k_attn_mass<true> : k_attn_mass<false>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(k, dim3(grid), dim3(320), smem, s, tmQ, tmK, p, n_ks);
+  return launch_pdl(k, dim3(grid), dim3(kAttnThreads), smem, s, tmQ, tmK, p, n_ks);
 }
 
 }  // namespace smoes
