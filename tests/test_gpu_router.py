@@ -3,7 +3,8 @@
 Small awkward cases cover several tiles with a ragged tail: T not a multiple of the 128/64-token
 tiles, d not a multiple of the 64/128-column blocks, E not a multiple of 16, one-token samples,
 non-consecutive bin maps, K = 1 and K = E, hard labels with an absent modality, renormalised
-top-k with an upstream weight gradient, and the fp32 path.
+top-k with an upstream weight gradient, the fp32 path, and the column splits of the two
+epilogue groups.
 """
 import numpy as np
 import pytest
@@ -34,6 +35,12 @@ CASES = {
     "single_token": (6, 1, 64, 16, 2, 4, [1], torch.bfloat16, True),
     "fp32": (7, 600, 128, 16, 2, 4, [600], torch.float32, True),
     "fp32_multi": (8, 333, 72, 32, 5, 8, [10, 200, 123], torch.float32, True),
+    # the two epilogue groups: a second group with one 16-column chunk and a partial 32-column
+    # staging block; consecutive bins that do not split at the half (group 0 takes all columns);
+    # the fp32 kernel with both groups holding columns
+    "split_odd_chunks": (9, 650, 256, 80, 5, 5, [330, 320], torch.bfloat16, True),
+    "contig_no_split": (10, 500, 192, 96, 6, 8, [250, 250], torch.bfloat16, False),
+    "fp32_split": (11, 300, 96, 64, 4, 8, [150, 150], torch.float32, True),
 }
 
 
