@@ -401,49 +401,83 @@ def main():
     ms_per_step = total_ms / args.steps
     value = job_rate(wl.T, world, ms_per_step)
 
-    # end to end through the public API: host inputs in pinned memory, copies inside the region
+    # end to end through the public API: every step's inputs come from pinned host memory and its
+    # loss goes back to the host, all inside the timed region. As in a training loop that
+    # prefetches, step i+1's inputs are copied on a second stream into the other of two device
+    # buffers while step i computes (a copy waits until the step that last used its buffer is
+    # done); the calls are the eager API calls. L2 is not flushed here: each step's inputs arrive
+    # by copy, as they would in deployment.
     e2e = None
     if not args.no_e2e:
         Xh = wl.X.pin_memory()
         Wh = wl.W.pin_memory()
         muh, varh = wl.mu.pin_memory(), wl.var.pin_memory()
-        lossh = torch.empty(1, dtype=torch.float32).pin_memory()
+        n_loss = args.steps + 3
+        lossh = torch.empty(n_loss, dtype=torch.float32).pin_memory()
         h2d = (Xh.numel() * Xh.element_size() + Wh.numel() * Wh.element_size() +
                muh.numel() * 4 + varh.numel() * 4)
         d2h = 4
-
+        bufs = [dict(X=X, W=W, mu=mu, var=var),
+                dict(X=torch.empty_like(X), W=torch.empty_like(W), mu=torch.empty_like(mu),
+                     var=torch.empty_like(var))]
         if use_attn:
             Qh, Kh = aw.Q.pin_memory(), aw.K.pin_memory()
             h2d += 2 * Qh.numel() * Qh.element_size()
+            bufs[0].update(Q=attn["Q"], K=attn["K"])
+            bufs[1].update(Q=torch.empty_like(attn["Q"]), K=torch.empty_like(attn["K"]))
+        cs = torch.cuda.Stream(device=dev)
+        main = torch.cuda.current_stream()
+        copied = [torch.cuda.Event(), torch.cuda.Event()]
+        done = [torch.cuda.Event(), torch.cuda.Event()]
 
-        def e2e_step():
-            X.copy_(Xh, non_blocking=True)
-            W.copy_(Wh, non_blocking=True)
-            mu.copy_(muh, non_blocking=True)
-            var.copy_(varh, non_blocking=True)
+        def issue_copy(i):
+            bb = bufs[i & 1]
+            with torch.cuda.stream(cs):
+                cs.wait_event(done[i & 1])             # the step that last read this buffer
+                bb["X"].copy_(Xh, non_blocking=True)
+                bb["W"].copy_(Wh, non_blocking=True)
+                bb["mu"].copy_(muh, non_blocking=True)
+                bb["var"].copy_(varh, non_blocking=True)
+                if use_attn:
+                    bb["Q"].copy_(Qh, non_blocking=True)
+                    bb["K"].copy_(Kh, non_blocking=True)
+                copied[i & 1].record(cs)
+
+        def compute(i):
+            bb = bufs[i & 1]
+            main.wait_event(copied[i & 1])
             if use_attn:
-                attn["Q"].copy_(Qh, non_blocking=True)
-                attn["K"].copy_(Kh, non_blocking=True)
-            for _, fn in parts:
-                fn()
-            lossh.copy_(r.loss, non_blocking=True)
+                a_args = dict(attn, Q=bb["Q"], K=bb["K"])
+                r.modality_score(bd.SMOES_SCORE_ATTN, Ma, attn=a_args)
+                r.forward_permute(bb["X"], bb["W"], M_in=Ma, bin_prob=False, is_vision=is_vis)
+                r.backward(bb["X"], bb["W"], Ma, dW, dX=dX, loss_scale=1e-4)
+            else:
+                r.forward_permute(bb["X"], bb["W"], mu=bb["mu"], var=bb["var"], tau=wl.tau,
+                                  bin_prob=False, is_vision=is_vis)
+                r.backward(bb["X"], bb["W"], r.M, dW, dX=dX, loss_scale=1e-4)
+            lossh[i:i + 1].copy_(r.loss, non_blocking=True)
+            done[i & 1].record(main)
 
-        for _ in range(3):
-            flush.zero_()
-            e2e_step()
+        def pipeline(n, first, start_ev=None):
+            if start_ev is not None:
+                cs.wait_event(start_ev)
+            issue_copy(first)
+            for i in range(first, first + n):
+                if i + 1 < first + n:
+                    issue_copy(i + 1)
+                compute(i)
+
+        pipeline(3, 0)                                 # warm-up
         torch.cuda.synchronize()
-        t_e2e = 0.0
-        for _ in range(args.steps):
-            flush.zero_()
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record()
-            e2e_step()
-            b.record()
-            b.synchronize()
-            t_e2e += a.elapsed_time(b)
-        t_e2e = max_over_ranks(t_e2e, world, dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(main)
+        pipeline(args.steps, 3, start_ev=a)
+        b.record(main)
+        b.synchronize()
+        t_e2e = max_over_ranks(a.elapsed_time(b), world, dev)
         e2e = {"value": job_rate(wl.T, world, t_e2e / args.steps), "unit": UNIT,
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "note": "inputs of step i+1 copied while step i computes (two device buffers)"}
 
     if rank != 0:
         if world > 1:
