@@ -288,7 +288,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   for (int e = 0; e < E && P->contig_bins; ++e) P->contig_bins = P->expert_bin[e] == e / P->N_B;
   P->dcoef = round_up(d.d, 256);
 
-  // token -> sample, 32-token groups -> pieces (one piece per (group, sample) pair)
+  // token -> sample, 128-token groups -> pieces (one piece per (group, sample) pair)
   P->n_groups = (T + kPieceTokens - 1) / kPieceTokens;
   P->token_sample.assign(std::max(T, 1), 0);
   for (int i = 0; i < B; ++i)
