@@ -72,14 +72,21 @@ WORKLOAD_TEXT = {
 
 
 def algorithmic(wl):
-    """Algorithmic bytes and flops of one step and of the backward call (the dominant launch)."""
+    """Algorithmic bytes and flops of one step, and bytes of its forward and backward calls."""
     T, d, E, k, K = wl.T, wl.d, wl.E, wl.k, wl.n_bins
     b = wl.X.element_size()
     per_token = 3 * d * b + 8 * k + 16 + 4 * k + 8 * min(k, K)
     step_bytes = T * per_token + E * d * (b + 4)
     step_flops = 6.0 * T * d * E
+    # forward + fused permutation: X read; top-k indices and weights, scores and permutation
+    # entries written; W read
+    fwd_bytes = T * (d * b + 8 * k + 8 + 8 * min(k, K)) + E * d * b
     bwd_bytes = T * (2 * d * b + 8) + E * d * (b + 4)        # X read, dX write, M read, W read, dW write
-    return step_bytes, step_flops, bwd_bytes, 4.0 * T * d * E
+    return step_bytes, step_flops, fwd_bytes, bwd_bytes
+
+
+# Special-function unit: 16 exp2 results per SM and clock (4 per sub-partition), 152 SMs.
+SFU_PER_SM_CLK = 16
 
 
 class ClockSampler:
@@ -148,9 +155,10 @@ class ClockSampler:
         return out
 
 
-def profile_traffic(kernel_file, workload):
-    """DRAM bytes per launch from a committed ncu summary, if it was taken on the current source."""
-    path = os.path.join(ROOT, "profiles", f"traffic_{workload}.json")
+def profile_traffic(kernel_file, workload, call):
+    """DRAM bytes per launch of a call (fwd / bwd) from a committed ncu summary, if it was taken on
+    the current source."""
+    path = os.path.join(ROOT, "profiles", f"traffic_{workload}_{call}.json")
     src = os.path.join(ROOT, "paper_2604_23996_gb300", "csrc", kernel_file)
     try:
         with open(path) as f:
@@ -396,7 +404,6 @@ def main():
     ms_per_step = total_ms / args.steps
     value = job_rate(wl.T, world, ms_per_step)
 
-    t_bwd = t_part["bwd"]
     total_ms = max_over_ranks(float(np.sum(t_step)), world, dev)
     ms_per_step = total_ms / args.steps
     value = job_rate(wl.T, world, ms_per_step)
@@ -485,17 +492,40 @@ def main():
         return
 
     hbm, tf_burst, tf_sus, peak_kind = peaks()
-    step_bytes, step_flops, bwd_bytes, bwd_flops = algorithmic(wl)
+    step_bytes, step_flops, fwd_bytes, bwd_bytes = algorithmic(wl)
     if use_attn:   # causal Q K^T of the attention score: B H S^2 hd flops; Q and K read once
         attn_flops = float(aw.B) * aw.H * aw.S * aw.S * aw.hd
         attn_bytes = 2.0 * aw.Q.numel() * aw.Q.element_size()
     else:
         attn_flops = attn_bytes = 0.0
-    bwd_ms = float(np.mean(t_bwd))
-    achieved = bwd_bytes / (bwd_ms * 1e-3) / 1e9
     t_roof = (max(step_bytes / (hbm * 1e9), step_flops / (tf_sus * 1e12)) +
               max(attn_bytes / (hbm * 1e9), attn_flops / (tf_sus * 1e12)))
-    traffic = profile_traffic("router_bwd.cu", args.config)
+    # roofline of every call of the step; `roofline` is the one of the longest call (the
+    # dominant kernel). The forward and backward are HBM-bound streams; the attention score
+    # evaluates one exponential per unmasked score on the special-function unit.
+    sm_mhz = float(clk.get("sm_max_mhz") or 2070.0)
+    rooflines = {}
+    for name in t_part:
+        ms = float(np.mean(t_part[name]))
+        if name == "attn":
+            n_exp = float(aw.B) * aw.H * aw.S * (aw.S + 1) / 2.0
+            peak = SFU_PER_SM_CLK * torch.cuda.get_device_properties(dev).multi_processor_count * sm_mhz * 1e-3
+            ach = n_exp / (ms * 1e-3) / 1e9
+            rooflines[name] = {"bound": "alu", "achieved": ach, "peak": peak, "unit": "Gexp/s",
+                               "frac": ach / peak, "traffic": None, "kernel": "k_attn_mass",
+                               "peak_source": "derived: 16 exp2 per SM and clock x SMs x max SM clock"}
+        else:
+            call = "fwd" if name.startswith("fwd") else "bwd"
+            by = fwd_bytes if call == "fwd" else bwd_bytes
+            ach = by / (ms * 1e-3) / 1e9
+            kern = ("smoes_router_fwd_permute (k_router_fwd_tc, one launch)" if call == "fwd" and not f32
+                    else "smoes_router_bwd (k_dz_prep + k_router_bwd_tc + k_dw_reduce)" if not f32
+                    else f"smoes_router_{call} (fp32 path)")
+            rooflines[name] = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                               "frac": ach / hbm, "bytes": by,
+                               "traffic": profile_traffic(f"router_{call}.cu", args.config, call),
+                               "kernel": kern, "peak_source": peak_kind}
+    dominant = max(t_part, key=lambda n: float(np.mean(t_part[n])))
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
@@ -511,10 +541,8 @@ def main():
                    "clocks": "nvidia-smi every 100 ms over a load window of ~0.5 s of steps "
                              "ending with the timed steps",
                    "parallelism": f"replicas x{world}"},
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm,
-                     "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
-                     "kernel": "smoes_router_bwd (k_router_bwd_tc + k_dw_reduce)",
-                     "peak_source": peak_kind},
+        "roofline": dict(rooflines[dominant], call=dominant),
+        "rooflines": rooflines,
         "step_roofline": {"t_roof_us": t_roof * 1e6, "t_step_us": ms_per_step * 1e3,
                           "frac": t_roof / (ms_per_step * 1e-3),
                           "bytes": step_bytes + attn_bytes, "flops": step_flops + attn_flops},
