@@ -1,0 +1,44 @@
+"""Host-side arithmetic of bench.py (no GPU): the algorithmic bytes and flops behind the
+roofline fractions, and the rule that an ncu traffic record counts only for the source it was
+taken on."""
+import hashlib
+import json
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+bench = pytest.importorskip("bench")
+from paper_2604_23996_gb300.workloads import config_workload  # noqa: E402
+
+
+def test_algorithmic_bytes_dsmoe_vlm():
+    # T = 16384, d = 2048, E = 64, k = 6, K = 8, bf16 (b = 2)
+    wl = config_workload("dsmoe_vlm")
+    step_bytes, step_flops, fwd_bytes, bwd_bytes = bench.algorithmic(wl)
+    T, d, E, k, K, b = 16384, 2048, 64, 6, 8, 2
+    assert fwd_bytes == T * (d * b + 8 * k + 8 + 8 * min(k, K)) + E * d * b == 69074944
+    assert bwd_bytes == T * (2 * d * b + 8) + E * d * (b + 4) == 135135232
+    assert step_bytes == T * (3 * d * b + 8 * k + 16 + 4 * k + 8 * min(k, K)) + E * d * (b + 4)
+    assert step_flops == 6.0 * T * d * E
+    # the step moves at least what its two calls move (the permutation reads the top-k again)
+    assert step_bytes >= fwd_bytes + bwd_bytes - E * d * b
+
+
+def test_traffic_record_only_for_its_source(tmp_path, monkeypatch):
+    prof = tmp_path / "profiles"
+    src_dir = tmp_path / "paper_2604_23996_gb300" / "csrc"
+    prof.mkdir()
+    src_dir.mkdir(parents=True)
+    src = src_dir / "router_fwd.cu"
+    src.write_text("// kernel v1\n")
+    sha = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    (prof / "traffic_w_fwd.json").write_text(json.dumps({"source_sha": sha, "dram_bytes_per_launch": 123.0}))
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.profile_traffic("router_fwd.cu", "w", "fwd") == 123.0
+    src.write_text("// kernel v2\n")                      # the kernel changed since the capture
+    assert bench.profile_traffic("router_fwd.cu", "w", "fwd") is None
+    assert bench.profile_traffic("router_fwd.cu", "other", "fwd") is None
