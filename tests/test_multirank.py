@@ -36,7 +36,7 @@ def _worker(rank, world, port, results):
 
 @pytest.mark.parametrize("world", [2])
 def test_ranks_take_the_slowest_time(world):
-    mgr = mp.Manager()
+    mgr = mp.get_context("spawn").Manager()       # no fork of a multi-threaded parent
     results = mgr.dict()
     mp.spawn(_worker, args=(world, _free_port(), results), nprocs=world, join=True)
     assert sorted(results.keys()) == list(range(world))
