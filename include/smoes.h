@@ -37,7 +37,7 @@ extern "C" {
 typedef enum {
   SMOES_OK = 0,
   SMOES_ERR_INVALID_ARG = -1,     /* bad size, pointer, map or offsets; nothing launched      */
-  SMOES_ERR_UNSUPPORTED = -2,     /* valid but outside what this build supports              */
+  SMOES_ERR_UNSUPPORTED = -2,     /* valid but outside what the library supports            */
   SMOES_ERR_ALIGNMENT = -3,       /* a pointer is not 16-byte aligned                        */
   SMOES_ERR_WORKSPACE = -4,       /* workspace missing or smaller than smoes_workspace_bytes */
   SMOES_ERR_CUDA = -5,            /* a CUDA runtime/driver call or a launch failed           */

@@ -7,8 +7,7 @@ table or helper with that path.
 
 Every function follows the paper ("Soft Modality-Guided Expert Specialization in MoE-VLMs")
 step by step, in float64, with numpy primitives (matmul, sort, log/exp) only. Where the paper
-is silent the reading used is stated in the docstring; the same readings are listed in
-DESIGN.md.
+is silent the reading used is stated in the function's docstring.
 
 Conventions
 -----------
