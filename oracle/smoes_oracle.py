@@ -388,3 +388,81 @@ def msi(expert_counts):
     share = C / C.sum(axis=1, keepdims=True)            # C_{m,e} / sum_e' C_{m,e'}
     Ct = share / share.sum(axis=0, keepdims=True)       # eq. (18)
     return float(np.mean(2.0 * np.abs(Ct[1] - 0.5)))    # eq. (19), text row
+
+
+# --------------------------------------------------------------------------------------------
+# Online statistics and momentum-adaptive binning (Secs. 3.2 and 3.3)
+# --------------------------------------------------------------------------------------------
+
+def gaussian_stats_empty(d):
+    """The empty state (N, S_mu, S_var) of the per-modality statistics: all zeros."""
+    return np.zeros(2), np.zeros((2, d)), np.zeros((2, d))
+
+
+def gaussian_stats_update(state, X, is_vision, beta):
+    """One step of the EMA variant of Welford's algorithm, eqs. (5)-(7), for both modalities.
+
+    state = (N [2], S_mu [2, d], S_var [2, d]) at step t-1; X [T, d]; is_vision [T] (hard labels:
+    T_m is the set of the batch's modality-m tokens); beta: the EMA decay. Returns the state at t:
+
+        N_t     = beta N_{t-1} + |T_m|                                                  (5)
+        S_mu,t  = beta S_mu,t-1 + |T_m| mu_{T_m}                                        (6)
+        S_var,t = beta S_var,t-1 + sum_{x in T_m} (x - mu_{T_m})^2
+                  + (mu_{T_m} - S_mu,t-1 / N_{t-1})^2 beta N_{t-1} |T_m| / (beta N_{t-1} + |T_m|)  (7)
+
+    with mu_{T_m} the batch mean of modality m. Readings: the last term of (7) is zero when
+    N_{t-1} = 0 (empty state: the factor is 0 and the previous mean undefined) or |T_m| = 0 (no
+    token of the modality in the batch: the batch mean undefined, the factor 0).
+    """
+    N0, Smu0, Svar0 = (_f64(a) for a in state)
+    X = _f64(X)
+    lab = np.asarray(is_vision)
+    N, Smu, Svar = np.empty(2), np.empty_like(Smu0), np.empty_like(Svar0)
+    for m, rows in enumerate((lab == 1, lab == 0)):       # row 0 vision, row 1 text
+        Xm = X[rows]
+        n = Xm.shape[0]
+        N[m] = beta * N0[m] + n
+        if n == 0:
+            Smu[m] = beta * Smu0[m]
+            Svar[m] = beta * Svar0[m]
+            continue
+        mu_b = Xm.mean(axis=0)
+        Smu[m] = beta * Smu0[m] + n * mu_b
+        Svar[m] = beta * Svar0[m] + np.sum((Xm - mu_b[None, :]) ** 2, axis=0)
+        if N0[m] > 0:
+            w = beta * N0[m] * n / (beta * N0[m] + n)
+            Svar[m] += (mu_b - Smu0[m] / N0[m]) ** 2 * w
+    return N, Smu, Svar
+
+
+def gaussian_stats(state):
+    """The distribution parameters of Sec. 3.2: mu_m = S_mu / N and var_m = S_var / N, [2, d]."""
+    N, Smu, Svar = (_f64(a) for a in state)
+    return Smu / N[:, None], Svar / N[:, None]
+
+
+def expert_load_ema(C_bar, C, beta):
+    """Eq. (10): C_bar_t = beta C_bar_{t-1} + (1 - beta) C, per modality and expert [2, E]."""
+    return beta * _f64(C_bar) + (1.0 - beta) * _f64(C)
+
+
+def text_bias(C_bar):
+    """Eq. (11): f_spec(e) = C_bar[text, e] / (C_bar[text, e] + C_bar[vision, e]), [E].
+
+    Reading: an expert with no load from either modality (0/0) is neutral, f = 1/2.
+    """
+    C_bar = _f64(C_bar)
+    tot = C_bar[0] + C_bar[1]
+    return np.where(tot > 0, C_bar[1] / np.where(tot > 0, tot, 1.0), 0.5)
+
+
+def adaptive_bins(f_spec, n_bins):
+    """Momentum-adaptive binning (Sec. 3.3): experts sorted by f_spec and cut into n_bins runs of
+    N_B = E / n_bins consecutive experts. Readings: ascending order (bin 0 holds the most
+    vision-biased experts), equal scores kept in expert-index order. Returns expert_bin [E]."""
+    f = _f64(f_spec)
+    E = f.shape[0]
+    order = np.argsort(f, kind="stable")
+    expert_bin = np.empty(E, dtype=np.int32)
+    expert_bin[order] = np.arange(E) // (E // n_bins)
+    return expert_bin
