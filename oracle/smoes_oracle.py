@@ -466,3 +466,75 @@ def adaptive_bins(f_spec, n_bins):
     expert_bin = np.empty(E, dtype=np.int32)
     expert_bin[order] = np.arange(E) // (E // n_bins)
     return expert_bin
+
+
+# --------------------------------------------------------------------------------------------
+# Bin-level load balance (Sec. 3.5)
+# --------------------------------------------------------------------------------------------
+
+def bin_balance_loss(g, topk_idx, expert_bin, n_bins):
+    """Bin-level load-balance loss of one layer, eq. (16):
+        L_bal = sum_k N_B sum_{e in B_k} f_e P_e,
+    with f_e and P_e taken over the tokens routed to bin B_k. Readings (the paper defers to the
+    load-balance terms of its preliminaries): U_k is the set of tokens with at least one of
+    their top-k experts in B_k; f_e = (selections of e) / (selections of all experts of B_k),
+    P_e = mean over j in U_k of g_je / sum_{e' in B_k} g_je' (the gate renormalised inside the
+    bin). Both sum to 1 over a bin, so a bin whose load is spread evenly gives 1. A bin that no
+    token selects contributes 0. With one bin this is the standard loss N_e sum_e f_e P_e of the
+    preliminaries (f_e over all selections, P_e the mean gate).
+
+    g [T, E] softmax scores, topk_idx [T, k] -> (L, dict(f [E], P [E], used [K] bool)).
+    """
+    g = _f64(g)
+    T, E = g.shape
+    eb = np.asarray(expert_bin)
+    N_B = E // n_bins
+    sel = np.zeros((T, E), dtype=bool)
+    sel[np.arange(T)[:, None], np.asarray(topk_idx)] = True
+    f = np.zeros(E)
+    P = np.zeros(E)
+    used = np.zeros(n_bins, dtype=bool)
+    L = 0.0
+    for k in range(n_bins):
+        members = np.nonzero(eb == k)[0]
+        U = sel[:, members].any(axis=1)                       # tokens routed to bin k
+        n_sel = sel[:, members].sum()
+        if n_sel == 0:
+            continue
+        used[k] = True
+        f[members] = sel[:, members].sum(axis=0) / n_sel
+        gk = g[U][:, members]
+        P[members] = np.mean(gk / gk.sum(axis=1, keepdims=True), axis=0)
+        L += N_B * float(np.sum(f[members] * P[members]))
+    return L, dict(f=f, P=P, used=used)
+
+
+def bin_balance_grad_logits(z, topk_idx, expert_bin, n_bins, scale):
+    """Gradient of scale * L_bal (eq. 16) at the gate logits z [T, E], with the routing
+    fractions f_e held constant (they are counts; the gradient flows through P_e only, as for
+    the standard load-balance loss). With h_je = g_je / G_jk, G_jk = sum_{e' in B_k} g_je' for a
+    token j in U_k and e in B_k:
+        dL/dg_je = N_B / |U_k| * (f_e - sum_{e' in B_k} f_e' h_je') / G_jk,
+    then through the softmax: dz_je = g_je (dL/dg_je - sum_e' g_je' dL/dg_je')."""
+    z = _f64(z)
+    g = softmax_gate(z)
+    T, E = g.shape
+    eb = np.asarray(expert_bin)
+    N_B = E // n_bins
+    _, parts = bin_balance_loss(g, topk_idx, expert_bin, n_bins)
+    f = parts["f"]
+    sel = np.zeros((T, E), dtype=bool)
+    sel[np.arange(T)[:, None], np.asarray(topk_idx)] = True
+    dg = np.zeros((T, E))
+    for k in range(n_bins):
+        if not parts["used"][k]:
+            continue
+        members = np.nonzero(eb == k)[0]
+        U = sel[:, members].any(axis=1)
+        gk = g[U][:, members]
+        G = gk.sum(axis=1, keepdims=True)
+        h = gk / G
+        fk = f[members][None, :]
+        dg[np.ix_(np.nonzero(U)[0], members)] = N_B / U.sum() * (fk - np.sum(fk * h, axis=1, keepdims=True)) / G
+    dg *= scale
+    return g * (dg - np.sum(g * dg, axis=1, keepdims=True))
