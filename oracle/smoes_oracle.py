@@ -111,6 +111,38 @@ def attention_vision_mass(Q, K, m_keys, sm_scale, causal=True, key_bias=None, qu
     return np.array([one_query(int(b), int(j)) for b, j in queries])
 
 
+def attention_forward_with_mass(Q, K, V, m_keys, sm_scale, causal=True, key_bias=None):
+    """Causal attention output and the aggregated vision score in one pass, the fused form of
+    eqs. (2)-(3): the score is attention with the carried score m as one more value column, so
+    O_ext = Attn [V | m] gives the layer's output (first dv columns) and, averaged over heads, its
+    last column is Mtilde_v. Grouped-query attention: K and V may have Hkv = H / G heads; query
+    head h reads key/value head h // G.
+
+    Q [B, H, S, hd]; K [B, Hkv, S, hd]; V [B, Hkv, S, dv]; m_keys [B, S]; key_bias [B, S] or None.
+    Returns (O [B, H, S, dv], Mtilde_v [B, S]).
+    """
+    Q, K, V, m_keys = _f64(Q), _f64(K), _f64(V), _f64(m_keys)
+    B, H, S, _ = Q.shape
+    Hkv = K.shape[1]
+    G = H // Hkv
+    bias = np.zeros((B, S)) if key_bias is None else _f64(key_bias)
+    O = np.empty((B, H, S, V.shape[3]))
+    mass = np.zeros((B, S))
+    for b in range(B):
+        for h in range(H):
+            hk = h // G
+            logits = sm_scale * (Q[b, h] @ K[b, hk].T) + bias[b][None, :]
+            if causal:
+                logits = np.where(np.tri(S, dtype=bool), logits, -np.inf)
+            logits = logits - logits.max(axis=1, keepdims=True)
+            w = np.exp(logits)
+            w = w / w.sum(axis=1, keepdims=True)
+            ext = w @ np.concatenate([V[b, hk], m_keys[b][:, None]], axis=1)
+            O[b, h] = ext[:, :-1]
+            mass[b] += ext[:, -1] / H
+    return O, mass
+
+
 def residual_score_update(M_tilde, M_prev, xattn_norm, x_norm):
     """Residual-weighted score update, eq. (4):
     M_next = (|x_attn| * Mtilde + |x| * M_prev) / (|x_attn| + |x|), per token and modality.
