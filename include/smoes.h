@@ -56,9 +56,11 @@ typedef enum {
 typedef struct smoes_plan_s* smoes_plan;
 
 /* Shape and routing metadata of one router layer (Secs. 3.1, 3.3).
- *   T >= 0 tokens; d hidden size (d % 8 == 0, d >= 8); E routed experts (1..256);
+ *   T tokens (0..2^20); d hidden size (d % 8 == 0, d >= 8); E routed experts (1..128 for
+ *   SMOES_BF16 plans, 1..64 for SMOES_F32 plans; larger E returns SMOES_ERR_UNSUPPORTED);
  *   k top-k (1..16, k <= E); n_bins bins (1..32, E % n_bins == 0, E / n_bins <= 32);
- *   n_samples >= 1 when T > 0 (0 when T == 0).
+ *   n_samples >= 1 when T > 0 (0 when T == 0). Every plan this call accepts runs in every
+ *   call below (the attention score adds its own limit on the head size).
  *   sample_offsets_host [n_samples+1]: 0 = o_0 < o_1 < ... < o_B = T (no empty sample).
  *   expert_bin_host [E]: bin of each expert, each bin holding exactly E / n_bins experts.
  *   renorm_topk: 0 -> top-k weights are the softmax scores; 1 -> renormalised over the top-k.
@@ -86,7 +88,8 @@ typedef struct {
 
 /* Attention-accumulated score inputs, eqs. (2)-(4).
  *   Q, K [B, H, S, hd] bf16 with B * S == T (token b*S + j is query j of sequence b);
- *   hd % 16 == 0, hd <= 256.
+ *   hd == 128 (other head sizes return SMOES_ERR_UNSUPPORTED); 1 <= H <= attn_max_heads of
+ *   the plan (else SMOES_ERR_WORKSPACE).
  *   Exactly one of is_vision ([T] uint8, the hard labels of eq. (2)) or m_prev ([T] float32,
  *   the previous layer's vision score) gives the score carried by every key.
  *   key_bias [T] float32 or NULL: added to the logit of key j of its sequence.
@@ -126,6 +129,13 @@ size_t smoes_workspace_bytes(smoes_plan plan);
 smoes_status smoes_workspace_init(smoes_plan plan, void* ws, size_t ws_bytes, cudaStream_t stream);
 
 const char* smoes_status_string(smoes_status status);
+
+/* Limit, in nanoseconds, of every bounded wait inside the plan's kernels (pipeline barriers,
+ * the grid barriers of the cooperative launches, tickets). A wait that exceeds it records
+ * SMOES_ERR_DEVICE_TIMEOUT in the workspace status word and the kernel returns without
+ * finishing its outputs. The default is 2 s; limit_ns == 0 restores it. Applies to calls made
+ * after it returns. */
+smoes_status smoes_plan_set_wait_limit(smoes_plan plan, uint64_t limit_ns);
 
 /* Synchronises `stream`, reads the workspace status word and returns SMOES_OK,
  * SMOES_ERR_DATA or SMOES_ERR_DEVICE_TIMEOUT. *n_absent_modality (optional) receives how many
@@ -203,15 +213,17 @@ smoes_status smoes_bin_permute(smoes_plan plan, const int32_t* topk_idx, const i
 
 /* (4b) The bin permutation of (4) without a workspace, for callers that cannot allocate device
  *   memory. The paper has no counterpart; this is a deployment convenience. Some callers cannot
- *   call cudaMalloc: code that runs while a CUDA graph is being captured or that must not trigger
- *   the implicit device synchronisation cudaMalloc can cause, serving runtimes whose device memory
- *   is planned up front by an arena that hands out no further blocks, and plug-ins that receive
- *   only their input and output buffers from a host framework.
+ *   call cudaMalloc: serving runtimes whose device memory is planned up front by an arena that
+ *   hands out no further blocks, plug-ins that receive only their input and output buffers from a
+ *   host framework, and latency-critical loops that must not risk the implicit device-wide
+ *   synchronisation an allocation can cause.
  *   Same arguments and results as smoes_bin_permute, minus the workspace. The scratch it needs
  *   (about 130 KB: block counts for up to 1024 permutation blocks x 32 bins, the bin
  *   map of up to 256 experts, a status word) is a fixed array inside the library, one per device
  *   that loads it, held until the process exits; this covers every plan smoes_plan_create
- *   accepts, and larger shapes return SMOES_ERR_UNSUPPORTED.
+ *   accepts, and larger shapes return SMOES_ERR_UNSUPPORTED. Each call first writes the plan's
+ *   bin map (passed to a small kernel by value) into that array and clears its status and
+ *   barrier words, on the given stream.
  *   The first call on a device looks up that array's device address (once per device); make that
  *   first call before any stream capture. Every call shares the one array (each call rewrites
  *   what it reads), so calls that overlap on the GPU, on any stream, race: order them. Device-side

@@ -63,6 +63,7 @@ _sig = {
     "smoes_workspace_bytes": (_sz, [_vp]),
     "smoes_workspace_init": (_i, [_vp, _vp, _sz, _vp]),
     "smoes_status_string": (C.c_char_p, [_i]),
+    "smoes_plan_set_wait_limit": (_i, [_vp, C.c_uint64]),
     "smoes_read_device_status": (_i, [_vp, _vp, _vp, C.POINTER(C.c_int32)]),
     "smoes_modality_score": (_i, [_vp, _i, C.POINTER(ScoreArgs), _vp, _vp, _sz, _vp]),
     "smoes_router_fwd": (_i, [_vp, _vp, _vp, _vp, C.POINTER(GaussArgs), _vp, _vp, _vp, _vp, _vp,
@@ -114,6 +115,10 @@ def smoes_plan_create(T, d, E, k, n_bins, sample_offsets, expert_bin, dtype, ren
     h = C.c_void_p()
     code = _lib.smoes_plan_create(C.byref(desc), C.byref(h))
     return code, h
+
+
+def smoes_plan_set_wait_limit(plan, limit_ns: int) -> int:
+    return _lib.smoes_plan_set_wait_limit(plan, int(limit_ns))
 
 
 def smoes_plan_destroy(plan):

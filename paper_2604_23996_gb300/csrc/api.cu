@@ -43,6 +43,7 @@ struct smoes_plan_s {
   int perm_nblocks = 0;
   int dcoef = 256;       // Gaussian coefficient vectors padded to 256 features
   bool contig_bins = false;
+  uint64_t limit_ns = kWaitLimitNs;   // bounded device waits
   std::vector<int32_t> offsets, expert_bin, expert_slot, token_sample, piece_base, sample_pieces;
   Layout L{};
 };
@@ -196,7 +197,7 @@ smoes_status router_fwd(smoes_plan P, const void* X, const void* W, const float*
   p.joint = joint;
   p.mi = mi;
   p.loss = loss;
-  p.limit_ns = kWaitLimitNs;
+  p.limit_ns = P->limit_ns;
   if (perm) {
     p.perm = *perm;
     p.perm.cta_counts = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + P->L.fperm);
@@ -252,6 +253,9 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
     return SMOES_ERR_UNSUPPORTED;
   if (d.T == 0 ? d.n_samples != 0 : d.n_samples < 1) return SMOES_ERR_INVALID_ARG;
   if (d.T > 0 && (!d.sample_offsets_host || !d.expert_bin_host)) return SMOES_ERR_INVALID_ARG;
+  // what every later call can run: the backward's accumulators (bf16: E_pad <= 128 TMEM columns
+  // per d-block; fp32: 64 logits per thread)
+  if (d.E > (d.dtype == SMOES_BF16 ? kMaxExpertsBf16 : kMaxExpertsF32)) return SMOES_ERR_UNSUPPORTED;
   if (d.T > (1 << 20)) return SMOES_ERR_UNSUPPORTED;          // permutation: <= 1024 blocks
   if (static_cast<long long>(d.T) * d.d > (1ll << 40)) return SMOES_ERR_UNSUPPORTED;
 
@@ -360,6 +364,12 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
 
 void smoes_plan_destroy(smoes_plan plan) { delete plan; }
 
+smoes_status smoes_plan_set_wait_limit(smoes_plan plan, uint64_t limit_ns) {
+  if (!plan) return SMOES_ERR_INVALID_ARG;
+  plan->limit_ns = limit_ns ? limit_ns : kWaitLimitNs;
+  return SMOES_OK;
+}
+
 size_t smoes_workspace_bytes(smoes_plan plan) { return plan ? plan->L.total : 0; }
 
 smoes_status smoes_workspace_init(smoes_plan P, void* ws, size_t ws_bytes, cudaStream_t stream) {
@@ -454,7 +464,7 @@ smoes_status smoes_modality_score(smoes_plan P, smoes_score_mode mode, const smo
     p.status = v.status;
     p.n_qtiles = (a.S + 127) / 128;
     p.n_items = a.B * p.n_qtiles * a.H;
-    p.limit_ns = kWaitLimitNs;
+    p.limit_ns = P->limit_ns;
     CUtensorMap tq, tk;
     const uint64_t rows = static_cast<uint64_t>(a.B) * a.H * a.S;
     if (!encode_bf16_2d(&tq, a.Q, rows, a.hd, 128, 64, true) ||
@@ -545,7 +555,7 @@ smoes_status smoes_router_bwd(smoes_plan P, const void* X, const void* W, const 
   p.slices = P->bwd_slices;
   p.slice_width = P->bwd_slice_width;
   p.n_tiles = P->bwd_tiles;
-  p.limit_ns = kWaitLimitNs;
+  p.limit_ns = P->limit_ns;
   cudaError_t e;
   if (d.dtype == SMOES_BF16) {
     const int E_pad = round_up(d.E, 64);
@@ -605,7 +615,7 @@ smoes_status smoes_bin_permute(smoes_plan P, const int32_t* topk_idx, const int3
   p.status = v.status;
   p.n_blocks = P->perm_nblocks;
   p.rounds = perm_rounds(d.T, d.k);
-  p.limit_ns = kWaitLimitNs;
+  p.limit_ns = P->limit_ns;
   return cuda_status(launch_bin_permute(p, stream));
 }
 
@@ -632,14 +642,9 @@ extern "C" smoes_status smoes_bin_permute_noalloc(smoes_plan P, const int32_t* t
   StaticPermScratch* sp = nullptr;
   cudaError_t e = static_perm_scratch(&sp);
   if (e != cudaSuccess) return SMOES_ERR_CUDA;
-  // the plan's bin map and slots into the scratch; the status and barrier words start at zero
-  e = cudaMemcpyAsync(sp->expert_bin, P->expert_bin.data(), sizeof(int32_t) * d.E,
-                      cudaMemcpyHostToDevice, stream);
-  if (e == cudaSuccess)
-    e = cudaMemcpyAsync(sp->expert_slot, P->expert_slot.data(), sizeof(int32_t) * d.E,
-                        cudaMemcpyHostToDevice, stream);
-  if (e == cudaSuccess) e = cudaMemsetAsync(sp->status, 0, sizeof(sp->status), stream);
-  if (e == cudaSuccess) e = cudaMemsetAsync(sp->sync, 0, sizeof(sp->sync), stream);
+  // the plan's bin map and slots into the scratch (kernel parameters, by value: nothing on the
+  // host is read after this call returns); the status and barrier words start at zero
+  e = launch_static_perm_prep(sp, P->expert_bin.data(), P->expert_slot.data(), d.E, stream);
   if (e != cudaSuccess) return SMOES_ERR_CUDA;
   PermParams p{};
   p.T = d.T;
@@ -661,6 +666,6 @@ extern "C" smoes_status smoes_bin_permute_noalloc(smoes_plan P, const int32_t* t
   p.status = sp->status;
   p.n_blocks = P->perm_nblocks;
   p.rounds = perm_rounds(d.T, d.k);
-  p.limit_ns = kWaitLimitNs;
+  p.limit_ns = P->limit_ns;
   return cuda_status(launch_bin_permute(p, stream));
 }

@@ -245,6 +245,40 @@ cudaError_t static_perm_scratch(StaticPermScratch** out) {
   return cudaSuccess;
 }
 
+// The plan's bin map and slots travel to the device as kernel parameters (2 KB, by value, so no
+// host buffer is referenced once the launch returns); one block writes them into the fixed
+// scratch and clears its status and grid-barrier words.
+struct StaticPermMaps {
+  int32_t expert_bin[kMaxExperts];
+  int32_t expert_slot[kMaxExperts];
+  int E;
+};
+
+__global__ void __launch_bounds__(kPermThreads) k_static_perm_prep(const StaticPermMaps m,
+                                                                    StaticPermScratch* sp) {
+  for (int e = threadIdx.x; e < m.E; e += kPermThreads) {
+    sp->expert_bin[e] = m.expert_bin[e];
+    sp->expert_slot[e] = m.expert_slot[e];
+  }
+  if (threadIdx.x < 4) {
+    sp->status[threadIdx.x] = 0u;
+    sp->sync[threadIdx.x] = 0u;
+  }
+}
+
+cudaError_t launch_static_perm_prep(StaticPermScratch* sp, const int32_t* expert_bin,
+                                    const int32_t* expert_slot, int E, cudaStream_t s) {
+  if (E < 1 || E > kMaxExperts) return cudaErrorInvalidValue;
+  StaticPermMaps m;
+  for (int e = 0; e < kMaxExperts; ++e) {
+    m.expert_bin[e] = e < E ? expert_bin[e] : 0;
+    m.expert_slot[e] = e < E ? expert_slot[e] : 0;
+  }
+  m.E = E;
+  k_static_perm_prep<<<1, kPermThreads, 0, s>>>(m, sp);
+  return cudaGetLastError();
+}
+
 template <class F>
 cudaError_t with_kernel(int k, F&& f) {
   if (k <= 2) return f(k_perm<2>);

@@ -12,7 +12,9 @@ namespace smoes {
 
 constexpr int kMaxTopK = 16;
 constexpr int kMaxBins = 32;
-constexpr int kMaxExperts = 256;
+constexpr int kMaxExperts = 256;           // bound of the permutation and metadata arrays
+constexpr int kMaxExpertsBf16 = 128;       // experts a bf16 plan accepts
+constexpr int kMaxExpertsF32 = 64;         // experts an fp32 plan accepts
 constexpr int kPieceTokens = 128;          // tokens per partial-sum "piece" (one forward tile)
 constexpr uint32_t kStatusData = 1u;       // status word bits
 constexpr uint32_t kStatusTimeout = 2u;
@@ -177,6 +179,10 @@ struct StaticPermScratch {
 };
 // Device address of that array on the current device (resolved once per device).
 cudaError_t static_perm_scratch(StaticPermScratch** out);
+// Writes a plan's bin map and slots (host arrays of E entries, passed to the kernel by value)
+// into that array and clears its status and barrier words, in stream order.
+cudaError_t launch_static_perm_prep(StaticPermScratch* sp, const int32_t* expert_bin,
+                                    const int32_t* expert_slot, int E, cudaStream_t s);
 
 // ------------------------------------------------------------------ launchers (in .cu files)
 // Every kernel of the library is launched with programmatic stream serialization: its CTAs may

@@ -62,10 +62,34 @@ def test_plan_create_ok_and_workspace_size(bd):
     (dict(expert_bin=np.arange(16) // 4 + 1), -1),           # bin out of range
     (dict(n_bins=64, E=64, expert_bin=np.arange(64)), -2),   # more than 32 bins
     (dict(k=0), -1),
+    # the limits every later call can run: E <= 128 (bf16), E <= 64 (fp32), T <= 2^20
+    (dict(E=256, k=8, n_bins=8, expert_bin=np.arange(256) // 32), -2),
+    (dict(E=136, k=8, n_bins=8, expert_bin=np.arange(136) // 17), -2),
+    (dict(E=128, k=8, n_bins=16, expert_bin=np.arange(128) // 8, dtype=0), -2),
+    (dict(T=(1 << 20) + 1, sample_offsets=[0, (1 << 20) + 1]), -2),
 ])
 def test_plan_create_rejects(bd, kw, code):
     got, plan = _plan(bd, **kw)
     assert got == code
+
+
+@pytest.mark.parametrize("kw", [
+    dict(E=128, k=8, n_bins=16, expert_bin=np.arange(128) // 8),            # largest bf16 plan
+    dict(E=64, k=6, n_bins=8, expert_bin=np.arange(64) // 8, dtype=0),      # largest fp32 plan
+    dict(T=1 << 20, sample_offsets=[0, 1 << 19, 1 << 20]),                  # largest batch
+])
+def test_plan_create_accepts_the_limits(bd, kw):
+    got, plan = _plan(bd, **kw)
+    assert got == 0
+    bd.smoes_plan_destroy(plan)
+
+
+def test_wait_limit_setter(bd):
+    code, plan = _plan(bd)
+    assert bd.smoes_plan_set_wait_limit(plan, 1000) == 0
+    assert bd.smoes_plan_set_wait_limit(plan, 0) == 0        # back to the default
+    assert bd.smoes_plan_set_wait_limit(None, 10) == -1
+    bd.smoes_plan_destroy(plan)
 
 
 def test_empty_batch_plan(bd):

@@ -2,9 +2,12 @@
 
 The GPU runs each workload once at full size; the fp64 oracle is evaluated sample by sample
 (samples are independent in eqs. 12-15; dW is the sum of the per-sample contributions), so host
-memory stays small. For the attention workload the score is checked on 64 seeded query rows
-(the full fp64 attention is ~3e11 flops), and its router stage runs at full size with the hard
-labels (the layer-0 score of eq. 2) as the provided scores.
+memory stays small. Every workload also runs in its aligned variant (tau = 1, bins tilted by
+modality), where the MI is far above the absolute floor of the scalar check. For the attention
+workload the score is compared on every query and head of the first and the last sequence
+(2 of 8 whole sequences; the full fp64 attention of all eight is ~5e11 flops), and its router
+stage runs at full size twice: with the hard labels (the layer-0 score of eq. 2) and with the
+GPU's own attention score as the provided scores (the score-to-router chain end to end).
 """
 import numpy as np
 import pytest
@@ -143,9 +146,10 @@ def test_fullsize_fused_equals_separate(bd):
         np.testing.assert_array_equal(np.asarray(a[key]), np.asarray(b[key]), err_msg=key)
 
 
-def test_fullsize_aligned_variant(bd):
+@pytest.mark.parametrize("key", ["tiny_fp32", "dsmoe_vlm", "small_hidden", "large_fine"])
+def test_fullsize_aligned_variant(bd, key):
     # same shapes, tau = 1 and bins tilted by modality: the MI is far from zero
-    wl = config_workload("dsmoe_vlm", aligned=True)
+    wl = config_workload(key, aligned=True)
     g = _run_full(bd, wl)
     _check_per_sample(wl, g)
     assert g["mi"].min() > 1e-6          # far above the 1e-9 absolute floor of the MI check
@@ -161,15 +165,21 @@ def test_fullsize_attention_workload(bd):
                 is_vision=torch.from_numpy(aw.is_vision).cuda())
     r.modality_score(bd.SMOES_SCORE_ATTN, M, attn=attn)
     assert r.device_status()[0] == 0
-    got = M.cpu().numpy()[:, 0].reshape(aw.B, aw.S)
-    rng = np.random.default_rng(77)
-    rows = np.stack([rng.integers(0, aw.B, 64), rng.integers(0, aw.S, 64)], axis=1)
+    Mg = M.cpu().numpy()
+    got = Mg[:, 0].reshape(aw.B, aw.S)
+    np.testing.assert_array_equal(Mg[:, 1], (1.0 - Mg[:, 0]).astype(np.float32))
     m = aw.is_vision.reshape(aw.B, aw.S).astype(np.float64)
-    ref = O.attention_vision_mass(aw.Q.double().numpy(), aw.K.double().numpy(), m, aw.sm_scale, True,
-                                  aw.key_bias.reshape(aw.B, aw.S), queries=rows)
-    assert_tensor_close(got[rows[:, 0], rows[:, 1]], ref, "attention vision mass (sampled rows)")
+    bias = aw.key_bias.reshape(aw.B, aw.S)
+    Qd, Kd = aw.Q, aw.K
+    for b in (0, aw.B - 1):                  # every query of every head of two whole sequences
+        ref = O.attention_vision_mass(Qd[b:b + 1].double().numpy(), Kd[b:b + 1].double().numpy(),
+                                      m[b:b + 1], aw.sm_scale, True, bias[b:b + 1])[0]
+        assert_tensor_close(got[b], ref, f"attention vision mass, sequence {b} (all queries)")
     # the router stage of this workload at full size, fed the layer-0 hard labels
     wl = config_workload("attn_router")
     Mh = np.stack([wl.is_vision, 1 - wl.is_vision], 1).astype(np.float32)
     g = _run_full(bd, wl, M_in=Mh)
     _check_per_sample(wl, g, M_provided=Mh)
+    # and fed the GPU's own attention score: the chain score -> router -> MI -> gradients
+    g = _run_full(bd, wl, M_in=np.ascontiguousarray(Mg))
+    _check_per_sample(wl, g, M_provided=Mg)
