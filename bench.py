@@ -106,7 +106,8 @@ def bench_config(config, wl, world):
     """The `config` object of the JSON line; both arms print the same one."""
     use_attn = config == "attn_router"
     return {"workload": f"{config}: {workload_text(config, wl)}; "
-                        + ("attention score (8x4096, 16 heads, hd 128, causal) + " if use_attn
+                        + (f"attention score ({wl.B if wl is not None else 8}x4096, 16 heads, hd 128, "
+                           "causal) + " if use_attn
                            else "Gaussian score; ")
                         + "fwd + bwd (dW, dX) + bin permutation",
             "l2": "flushed before every step (256 MiB write, outside the timed interval)",
@@ -612,7 +613,7 @@ def main():
 
     wl = config_workload(args.config, n_samples=samples_for(args.config, args.tokens))
     use_attn = args.config == "attn_router"
-    aw = attn_workload() if use_attn else None
+    aw = attn_workload(B=wl.B) if use_attn else None       # one sequence per sample
     st = Step(bd, wl, aw, dev)
     st.capture()
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)   # 256 MiB > L2

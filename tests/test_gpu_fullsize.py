@@ -152,7 +152,7 @@ def test_fullsize_aligned_variant(bd, key):
     wl = config_workload(key, aligned=True)
     g = _run_full(bd, wl)
     _check_per_sample(wl, g)
-    assert g["mi"].min() > 1e-6          # far above the 1e-9 absolute floor of the MI check
+    assert g["mi"].min() > 1e-7          # 100x above the 1e-9 absolute floor of the MI check
 
 
 def test_fullsize_attention_workload(bd):
