@@ -211,6 +211,39 @@ smoes_status smoes_bin_permute(smoes_plan plan, const int32_t* topk_idx, const i
                                int32_t* expert_counts, void* ws, size_t ws_bytes,
                                cudaStream_t stream);
 
+/* (5) Online statistics of the Gaussian modality score (Sec. 3.2, eqs. (5)-(7)): one step of the
+ *   EMA variant of Welford's algorithm for both modalities, in place.
+ *   X [T, d] (plan dtype); is_vision [T] uint8 (the hard labels: T_m is the batch's modality-m
+ *   tokens); beta in [0, 1] the EMA decay (the paper uses 0.99).
+ *   State (device, fp64, updated in place): N [2], S_mu [2, d], S_var [2, d] (row 0 vision,
+ *   row 1 text); all zeros is the empty state. Per modality m with n = |T_m|:
+ *     N = beta N + n;  S_mu = beta S_mu + n mu_T;
+ *     S_var = beta S_var + sum_{x in T_m} (x - mu_T)^2 + (mu_T - S_mu_old / N_old)^2 beta N_old n / (beta N_old + n),
+ *   the last term taken as 0 when N_old = 0 or n = 0 (mu_T the batch mean; see the paper for the
+ *   symbols). mu, var [2, d] float32 or NULL: S_mu / N and S_var / N after the update (the
+ *   statistics the next score uses; NaN for a modality never seen).
+ *   The batch sums are shifted by the previous mean (exact algebra, no cancellation); partial
+ *   sums are fp32 per block of rows and fp64 across blocks, in a fixed order (reproducible).
+ *   ws: the plan's workspace (per-block partial sums). */
+smoes_status smoes_gaussian_stats_update(smoes_plan plan, const void* X, const uint8_t* is_vision,
+                                         double beta, double* N, double* S_mu, double* S_var,
+                                         float* mu, float* var, void* ws, size_t ws_bytes,
+                                         cudaStream_t stream);
+
+/* (6) Momentum-adaptive binning (Sec. 3.3, eqs. (10)-(11)).
+ *   expert_counts [2, E] int32: this step's selections of each expert by the tokens of each hard
+ *   modality (the expert_counts output of (4)); C_bar [2, E] fp64, updated in place:
+ *   C_bar = beta C_bar + (1 - beta) C (eq. (10)). f_spec(e) = C_bar[text, e] / (C_bar[text, e] +
+ *   C_bar[vision, e]) (eq. (11); 1/2 for an expert with no load), written to f_spec [E] fp64
+ *   when not NULL. expert_bin [E] int32 receives the new map: experts sorted by ascending f_spec
+ *   (equal values in expert-index order) and cut into n_bins runs of E / n_bins, so bin 0 holds
+ *   the most vision-biased experts. All arithmetic is fp64 with separately rounded operations:
+ *   the map is reproducible bit for bit. The plan keeps its own map; a caller that adopts the
+ *   new one creates a plan from it (expert groupings change rarely: the loads are EMAs). */
+smoes_status smoes_adaptive_bins(smoes_plan plan, const int32_t* expert_counts, double beta,
+                                 double* C_bar, int32_t* expert_bin, double* f_spec,
+                                 cudaStream_t stream);
+
 /* (4b) The bin permutation of (4) without a workspace, for callers that cannot allocate device
  *   memory. The paper has no counterpart; this is a deployment convenience. Some callers cannot
  *   call cudaMalloc: serving runtimes whose device memory is planned up front by an arena that

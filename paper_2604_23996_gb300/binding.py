@@ -74,6 +74,9 @@ _sig = {
     "smoes_router_bwd": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _f, _vp, _i, _vp, _vp, _vp, _sz, _vp]),
     "smoes_bin_permute": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "smoes_bin_permute_noalloc": (_i, [_vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
+    "smoes_gaussian_stats_update": (_i, [_vp, _vp, _vp, C.c_double, _vp, _vp, _vp, _vp, _vp, _vp,
+                                         _sz, _vp]),
+    "smoes_adaptive_bins": (_i, [_vp, _vp, C.c_double, _vp, _vp, _vp, _vp]),
 }
 for _name, (_res, _args) in _sig.items():
     _fn = getattr(_lib, _name)
@@ -205,6 +208,18 @@ def smoes_bin_permute_noalloc(plan, topk_idx, home, is_vision, bin_offsets, perm
     return _lib.smoes_bin_permute_noalloc(plan, _p(topk_idx), _p(home), _p(is_vision),
                                           _p(bin_offsets), _p(perm_token), _p(perm_mask),
                                           _p(dispatch), _p(expert_counts), _stream(stream))
+
+
+def smoes_gaussian_stats_update(plan, X, is_vision, beta, N, S_mu, S_var, mu, var, ws,
+                                stream=None) -> int:
+    return _lib.smoes_gaussian_stats_update(plan, _p(X), _p(is_vision), float(beta), _p(N), _p(S_mu),
+                                            _p(S_var), _p(mu), _p(var), _p(ws),
+                                            ws.numel() * ws.element_size(), _stream(stream))
+
+
+def smoes_adaptive_bins(plan, expert_counts, beta, C_bar, expert_bin, f_spec=None, stream=None) -> int:
+    return _lib.smoes_adaptive_bins(plan, _p(expert_counts), float(beta), _p(C_bar), _p(expert_bin),
+                                    _p(f_spec), _stream(stream))
 
 
 # ----------------------------------------------------------------------------- convenience

@@ -24,7 +24,7 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 struct Layout {
   size_t status, sample_ticket, loss_ticket, offsets, token_sample, expert_bin, expert_slot,
       piece_base, sample_pieces, pieces, mi32, tabs, gsave, ginv, dw_part, dz_img, perm, attn_ticket, attn_part,
-      gcoef, perm_sync, fperm;
+      gcoef, perm_sync, fperm, stat_part, stat_nvis, stat_n0, f32_part, tile_ticket;
   size_t header_bytes;   // [0, header_bytes) is cleared by smoes_workspace_init
   size_t total;
 };
@@ -42,6 +42,7 @@ struct smoes_plan_s {
   int bwd_groups = 1, bwd_slices = 1, bwd_slice_width = 0;
   int perm_nblocks = 0;
   int dcoef = 256;       // Gaussian coefficient vectors padded to 256 features
+  int stat_blocks = 1;   // blocks of the statistics pass (one partial each)
   bool contig_bins = false;
   uint64_t limit_ns = kWaitLimitNs;   // bounded device waits
   std::vector<int32_t> offsets, expert_bin, expert_slot, token_sample, piece_base, sample_pieces;
@@ -203,11 +204,6 @@ smoes_status router_fwd(smoes_plan P, const void* X, const void* W, const float*
     p.perm.cta_counts = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + P->L.fperm);
     p.perm.sync = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + P->L.perm_sync);
   }
-  if (gauss && d.dtype == SMOES_F32) {
-    const cudaError_t e = launch_gauss_coef(gauss->mu, gauss->var, d.d, p.ws.dcoef, p.ws.gcoef,
-                                            p.ws.status, stream);
-    if (e != cudaSuccess) return SMOES_ERR_CUDA;
-  }
   if (d.dtype == SMOES_BF16) {
     p.n_tiles = (d.T + kFwdBM - 1) / kFwdBM;
     CUtensorMap tx, tw;
@@ -220,6 +216,9 @@ smoes_status router_fwd(smoes_plan P, const void* X, const void* W, const float*
     return cuda_status(launch_router_fwd_bf16(p, tx, tw, tma_g ? &tg : nullptr, P->n_sms, stream));
   }
   p.n_tiles = P->n_groups;
+  p.f32_chunks = f32_chunks(d.d);
+  p.f32_part = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + P->L.f32_part);
+  p.tile_ticket = reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(ws) + P->L.tile_ticket);
   return cuda_status(launch_router_fwd_f32(p, stream));
 }
 
@@ -338,6 +337,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.loss_ticket = take(sizeof(uint32_t) * 4);
   L.attn_ticket = take(sizeof(uint32_t) * (static_cast<size_t>(T) + 1));
   L.perm_sync = take(sizeof(uint32_t) * 4);
+  L.tile_ticket = take(sizeof(uint32_t) * static_cast<size_t>(std::max(P->n_groups, 1)));
   L.header_bytes = o;
   L.offsets = take(sizeof(int32_t) * (B + 1));
   L.token_sample = take(sizeof(int32_t) * std::max(T, 1));
@@ -357,6 +357,12 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.fperm = take(sizeof(int32_t) * static_cast<size_t>(std::max(P->n_sms, 1)) * K);   // per-CTA counts
   L.attn_part = take(sizeof(float) * static_cast<size_t>(T) * std::max(0, d.attn_max_heads));
   L.gcoef = take(sizeof(float) * (2 * static_cast<size_t>(P->dcoef) + P->dcoef / 256));
+  P->stat_blocks = std::max(1, std::min(2 * P->n_sms, (T + 63) / 64));
+  L.stat_part = take(sizeof(float) * 4 * static_cast<size_t>(P->stat_blocks) * d.d);
+  L.stat_nvis = take(sizeof(int32_t) * static_cast<size_t>(P->stat_blocks));
+  L.stat_n0 = take(sizeof(double) * 2);
+  L.f32_part = take(d.dtype == SMOES_F32 ? sizeof(float) * static_cast<size_t>(P->n_groups) *
+                                               f32_chunks(d.d) * (E + 1) * 128 : 0);
   L.total = o;
   *out = P;
   return SMOES_OK;
@@ -617,6 +623,58 @@ smoes_status smoes_bin_permute(smoes_plan P, const int32_t* topk_idx, const int3
   p.rounds = perm_rounds(d.T, d.k);
   p.limit_ns = P->limit_ns;
   return cuda_status(launch_bin_permute(p, stream));
+}
+
+smoes_status smoes_gaussian_stats_update(smoes_plan P, const void* X, const uint8_t* is_vision,
+                                         double beta, double* N, double* S_mu, double* S_var,
+                                         float* mu, float* var, void* ws, size_t ws_bytes,
+                                         cudaStream_t stream) {
+  if (!P) return SMOES_ERR_INVALID_ARG;
+  smoes_status st = check_ws(P, ws, ws_bytes);
+  if (st != SMOES_OK) return st;
+  const smoes_router_desc& d = P->desc;
+  if (!N || !S_mu || !S_var) return SMOES_ERR_INVALID_ARG;
+  if (d.T > 0 && (!X || !is_vision)) return SMOES_ERR_INVALID_ARG;
+  if (!(beta >= 0.0 && beta <= 1.0)) return SMOES_ERR_INVALID_ARG;
+  if ((X && !aligned16(X)) || !aligned16(N) || !aligned16(S_mu) || !aligned16(S_var) ||
+      (mu && !aligned16(mu)) || (var && !aligned16(var)))
+    return SMOES_ERR_ALIGNMENT;
+  uint8_t* b = static_cast<uint8_t*>(ws);
+  StatsParams p{};
+  p.T = d.T;
+  p.d = d.d;
+  p.G = P->stat_blocks;
+  p.X = X;
+  p.is_vision = is_vision;
+  p.beta = beta;
+  p.N = N;
+  p.S_mu = S_mu;
+  p.S_var = S_var;
+  p.mu_out = mu;
+  p.var_out = var;
+  p.part = reinterpret_cast<float*>(b + P->L.stat_part);
+  p.nvis = reinterpret_cast<int32_t*>(b + P->L.stat_nvis);
+  p.N0 = reinterpret_cast<double*>(b + P->L.stat_n0);
+  return cuda_status(launch_stats_update(p, d.dtype == SMOES_BF16, stream));
+}
+
+smoes_status smoes_adaptive_bins(smoes_plan P, const int32_t* expert_counts, double beta,
+                                 double* C_bar, int32_t* expert_bin, double* f_spec,
+                                 cudaStream_t stream) {
+  if (!P || !expert_counts || !C_bar || !expert_bin) return SMOES_ERR_INVALID_ARG;
+  if (!(beta >= 0.0 && beta <= 1.0)) return SMOES_ERR_INVALID_ARG;
+  if (!aligned16(expert_counts) || !aligned16(C_bar) || !aligned16(expert_bin) ||
+      (f_spec && !aligned16(f_spec)))
+    return SMOES_ERR_ALIGNMENT;
+  BinsParams p{};
+  p.E = P->desc.E;
+  p.N_B = P->N_B;
+  p.beta = beta;
+  p.counts = expert_counts;
+  p.C_bar = C_bar;
+  p.expert_bin = expert_bin;
+  p.f_spec = f_spec;
+  return cuda_status(launch_adaptive_bins(p, stream));
 }
 
 }  // extern "C"

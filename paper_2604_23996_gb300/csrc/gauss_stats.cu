@@ -29,7 +29,7 @@ namespace {
 
 constexpr int kStatThreads = 256;
 constexpr int kStatCols = 8 * kStatThreads;      // features per pass of a block (8 per thread)
-constexpr int kStatRowsInFlight = 4;             // rows loaded ahead per thread
+constexpr int kStatRowsInFlight = 8;             // rows loaded ahead per thread
 
 // Shift of feature i of modality m: the previous mean (fp32), or 0 for an empty state.
 __device__ __forceinline__ float stat_shift(const double* N0, const double* S_mu0, int d, int m, int i) {
@@ -37,21 +37,42 @@ __device__ __forceinline__ float stat_shift(const double* N0, const double* S_mu
   return n > 0.0 ? static_cast<float>(S_mu0[static_cast<size_t>(m) * d + i] / n) : 0.f;
 }
 
-// Eight consecutive features of row j as floats (bf16 or fp32 storage).
+// Eight consecutive features of a row: raw 16-byte words (bf16: one, fp32: two), loaded ahead
+// and widened to floats when they are used.
 template <bool kBf16>
-__device__ __forceinline__ void load8(const void* X, size_t off, float (&v)[8]) {
+struct Raw8 {
+  uint4 w[kBf16 ? 1 : 2];
+};
+
+template <bool kBf16>
+__device__ __forceinline__ void load_raw8(const void* X, size_t off, Raw8<kBf16>& r) {
   if (kBf16) {
-    const uint4 u = __ldg(reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(X) + off));
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    r.w[0] = __ldg(reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(X) + off));
+  } else {
+    const uint4* p = reinterpret_cast<const uint4*>(static_cast<const float*>(X) + off);
+    r.w[0] = __ldg(p);
+    r.w[kBf16 ? 0 : 1] = __ldg(p + 1);
+  }
+}
+
+template <bool kBf16>
+__device__ __forceinline__ void widen8(const Raw8<kBf16>& r, float (&v)[8]) {
+  if (kBf16) {
+    const uint32_t w[4] = {r.w[0].x, r.w[0].y, r.w[0].z, r.w[0].w};
 #pragma unroll
-    for (int r = 0; r < 4; ++r) {
-      v[2 * r] = __uint_as_float(w[r] << 16);
-      v[2 * r + 1] = __uint_as_float(w[r] & 0xffff0000u);
+    for (int q = 0; q < 4; ++q) {
+      v[2 * q] = __uint_as_float(w[q] << 16);
+      v[2 * q + 1] = __uint_as_float(w[q] & 0xffff0000u);
     }
   } else {
-    const float4* p = reinterpret_cast<const float4*>(static_cast<const float*>(X) + off);
-    const float4 a = __ldg(p), b = __ldg(p + 1);
-    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const uint4 u = r.w[kBf16 ? 0 : h];
+      v[4 * h] = __uint_as_float(u.x);
+      v[4 * h + 1] = __uint_as_float(u.y);
+      v[4 * h + 2] = __uint_as_float(u.z);
+      v[4 * h + 3] = __uint_as_float(u.w);
+    }
   }
 }
 
@@ -79,27 +100,24 @@ __global__ void __launch_bounds__(kStatThreads) k_stats_partial(const StatsParam
 #pragma unroll
     for (int q = 0; q < 8; ++q) s1[0][q] = s1[1][q] = s2[0][q] = s2[1][q] = 0.f;
     for (int j0 = r0; j0 < r1; j0 += kStatRowsInFlight) {
-      float v[kStatRowsInFlight][8];
+      Raw8<kBf16> raw[kStatRowsInFlight];
       int lab[kStatRowsInFlight];
 #pragma unroll
       for (int u = 0; u < kStatRowsInFlight; ++u) {
         const int j = j0 + u;
         lab[u] = j < r1 ? (__ldg(p.is_vision + j) ? 0 : 1) : -1;
-        if (act && j < r1) {
-          load8<kBf16>(p.X, static_cast<size_t>(j) * p.d + c, v[u]);
-        } else {
-#pragma unroll
-          for (int q = 0; q < 8; ++q) v[u][q] = 0.f;
-        }
+        if (act && j < r1) load_raw8<kBf16>(p.X, static_cast<size_t>(j) * p.d + c, raw[u]);
       }
 #pragma unroll
       for (int u = 0; u < kStatRowsInFlight; ++u) {
-        if (lab[u] < 0) continue;
+        if (lab[u] < 0 || !act) continue;
         if (c0 == 0 && threadIdx.x == 0 && lab[u] == 0) ++nv;
         const int m = lab[u];
+        float v[8];
+        widen8<kBf16>(raw[u], v);
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-          const float dv = v[u][q] - (m ? sh[1][q] : sh[0][q]);
+          const float dv = v[q] - (m ? sh[1][q] : sh[0][q]);
           if (m) {
             s1[1][q] += dv;
             s2[1][q] = fmaf(dv, dv, s2[1][q]);

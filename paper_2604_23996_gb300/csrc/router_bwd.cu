@@ -445,10 +445,13 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
 }
 
 // ------------------------------------------------------------------ FFMA backward (fp32)
-// One block per 64-token tile, all of d. dz for the tile is built in shared memory
-// (4 threads per token); then each thread owns one column per 256-column chunk, produces dX
-// for the tile and accumulates the tile's partial dW^T column in registers.
+// CTA (64-token tile, 128-feature chunk): dz of the tile's tokens into shared memory (4 threads
+// per token; every chunk of the tile forms the same dz, the first one writes dlogits), then
+// thread (feature c, half h) holds W[:, c] in registers and walks 32 of the tile's rows: dX[j, c]
+// = dz_j . W[:, c] and the partial dW[:, c] += dz_j x_jc. The two halves' dW partials are added
+// in shared memory and written once per tile; k_dw_reduce sums the tiles in order.
 constexpr int kF32MaxE = 64;
+constexpr int kF32Cols = 128;
 
 __global__ void __launch_bounds__(256)
 k_router_bwd_f32(const BwdParams p) {
@@ -457,9 +460,11 @@ k_router_bwd_f32(const BwdParams p) {
   pdl_trigger();
   const Dims& dm = p.dm;
   const int E = dm.E, K = dm.K, k = dm.k;
+  const int nck = (dm.d + kF32Cols - 1) / kF32Cols;
+  const int tile = blockIdx.x / nck, ck = blockIdx.x % nck;
   float* dzs = bs;                                   // [64][E+1]
+  float* dws = dzs + 64 * (E + 1);                   // [E][128] second half's dW partial
   const int t = threadIdx.x;
-  const int tile = blockIdx.x;
   {
     const int r = t >> 2, qd = t & 3;
     const int j = tile * 64 + r;
@@ -494,42 +499,61 @@ k_router_bwd_f32(const BwdParams p) {
         const float ge = g[e] * ginv;
         v = p.scale * ge * (u - part);
         if (has_up) v += ge * (upstream_at(up, k, e) - up.gdt);
-        if (p.dlogits) p.dlogits[static_cast<size_t>(j) * E + e] = v;
+        if (p.dlogits && ck == 0) p.dlogits[static_cast<size_t>(j) * E + e] = v;
       }
       dzs[r * (E + 1) + e] = v;
     }
   }
-  __syncthreads();
   const float* X = static_cast<const float*>(p.X);
   const float* W = static_cast<const float*>(p.W);
   float* dX = static_cast<float*>(p.dX);
-  const int rows = min(64, dm.T - tile * 64);
-  for (int c0 = 0; c0 < dm.d; c0 += 256) {
-    const int c = c0 + t;
-    if (c >= dm.d) break;
-    float wc[kF32MaxE], acc[kF32MaxE];
+  const int c = ck * kF32Cols + (t & 127), h = t >> 7;
+  const bool cin = c < dm.d;
+  float wc[kF32MaxE], acc[kF32MaxE];
 #pragma unroll
-    for (int e = 0; e < kF32MaxE; ++e) {
-      wc[e] = (e < E) ? W[static_cast<size_t>(e) * dm.d + c] : 0.f;
-      acc[e] = 0.f;
+  for (int e = 0; e < kF32MaxE; ++e) {
+    wc[e] = (e < E && cin) ? __ldg(W + static_cast<size_t>(e) * dm.d + c) : 0.f;
+    acc[e] = 0.f;
+  }
+  __syncthreads();
+  const int r0 = 32 * h;
+  const int rows = min(32, dm.T - tile * 64 - r0);
+  constexpr int kU = 8;                              // rows loaded ahead
+  for (int rb = 0; rb < rows; rb += kU) {
+    float x[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const size_t j = static_cast<size_t>(tile) * 64 + r0 + rb + u;
+      x[u] = (cin && rb + u < rows) ? __ldg(X + j * dm.d + c) : 0.f;
     }
-    for (int r = 0; r < rows; ++r) {
-      const size_t j = static_cast<size_t>(tile) * 64 + r;
-      const float x = X[j * dm.d + c];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      if (rb + u >= rows) break;
+      const float* zr = dzs + (r0 + rb + u) * (E + 1);
       float dx = 0.f;
 #pragma unroll
       for (int e = 0; e < kF32MaxE; ++e) {
         if (e < E) {
-          const float z = dzs[r * (E + 1) + e];
+          const float z = zr[e];
           dx = fmaf(z, wc[e], dx);
-          acc[e] = fmaf(z, x, acc[e]);
+          acc[e] = fmaf(z, x[u], acc[e]);
         }
       }
-      if (dX) dX[j * dm.d + c] = dx;
+      const size_t j = static_cast<size_t>(tile) * 64 + r0 + rb + u;
+      if (dX && cin) dX[j * dm.d + c] = dx;
     }
+  }
+  if (h == 1) {
 #pragma unroll
     for (int e = 0; e < kF32MaxE; ++e)
-      if (e < E) p.ws.dw_part[(static_cast<size_t>(tile) * E + e) * dm.d + c] = acc[e];
+      if (e < E) dws[e * kF32Cols + (t & 127)] = acc[e];
+  }
+  __syncthreads();
+  if (h == 0 && cin) {
+#pragma unroll
+    for (int e = 0; e < kF32MaxE; ++e)
+      if (e < E)
+        p.ws.dw_part[(static_cast<size_t>(tile) * E + e) * dm.d + c] = acc[e] + dws[e * kF32Cols + t];
   }
 }
 
@@ -623,8 +647,12 @@ cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, c
 
 cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s) {
   if (p.dm.E > kF32MaxE) return cudaErrorInvalidValue;
-  const size_t smem = sizeof(float) * 64 * (p.dm.E + 1);
-  return launch_pdl(k_router_bwd_f32, dim3(p.n_tiles), dim3(256), smem, s, p);
+  const size_t smem = sizeof(float) * (64 * (p.dm.E + 1) + static_cast<size_t>(p.dm.E) * kF32Cols);
+  cudaError_t e = cudaFuncSetAttribute(k_router_bwd_f32, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  const int nck = (p.dm.d + kF32Cols - 1) / kF32Cols;
+  return launch_pdl(k_router_bwd_f32, dim3(p.n_tiles * nck), dim3(256), smem, s, p);
 }
 
 cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s) {

@@ -1137,95 +1137,154 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
 }
 
 // ------------------------------------------------------------------ FFMA forward (fp32)
-// 128 tokens per block, 512 threads: thread (row r = t/4, quarter q = t%4) accumulates the
-// logits of experts e = q + 4i over d and a quarter of the Gaussian sum; threads 0..255 then
-// run the same two-group epilogue as the tensor-core path (logits read from shared memory).
+// The fp32 layers of the workloads are small (d ~ 512, E <= 64): one 128-token tile per CTA
+// would leave most SMs idle, so the hidden dimension is split as well. CTA (tile, chunk) stages
+// its 128 x 128 block of X and the matching [E, 128] block of W in shared memory (16-byte
+// asynchronous copies, all in flight at once), evaluates the chunk's Gaussian coefficients
+// (eqs. 8-9) and forms the partial logits and the partial log-likelihood difference of the
+// tile's rows over its 128 features. The last CTA of the tile to finish (a ticket) adds the
+// chunks' partials in chunk order (bitwise reproducible) and runs the same two-group epilogue as
+// the tensor-core path (logits read from shared memory).
 constexpr int kF32MaxE = 64;
+constexpr int kF32Cols = 128;                 // features per CTA
+constexpr int kF32XStride = kF32Cols + 4;     // row stride of the staged X block (floats)
 
 __host__ __device__ inline size_t f32_smem_floats(const Dims& dm) {
   const int E16 = round_up(dm.E, 16);
-  const int dpad = round_up(dm.d, 32);
-  return 128 * 33 + static_cast<size_t>(dm.E) * 33 + 128 * static_cast<size_t>(E16 + 1) + 2 * dpad +
-         epi_smem_floats(dm.K) + 128;
+  const size_t xs = static_cast<size_t>(kF32Cols) * kF32XStride;
+  const size_t zs = 128 * static_cast<size_t>(E16 + 1);
+  return (xs > zs ? xs : zs) + static_cast<size_t>(dm.E) * kF32Cols + 3 * kF32Cols + 8 +
+         epi_smem_floats(dm.K) + 3 * 128 + 8;
+}
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool in) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(in ? 16 : 0) : "memory");
 }
 
 template <bool kGauss, int KM>
-__global__ void __launch_bounds__(512)
+__global__ void __launch_bounds__(256)
 k_router_fwd_f32(const FwdParams p) {
   extern __shared__ float fs[];
   const Dims& dm = p.dm;
   const int E = dm.E, d = dm.d;
   const int E16 = round_up(E, 16);
-  const int dpad = round_up(d, 32);
-  float* xs = fs;                          // [128][33]
-  float* wsm = xs + 128 * 33;              // [E][33]
-  float* zs = wsm + E * 33;                // [128][E16 + 1]
-  float* ga = zs + 128 * (E16 + 1);        // [dpad]
-  float* gb = ga + dpad;                   // [dpad]
-  float* epi = gb + dpad;                  // epilogue tables
-  float* dll_s = epi + epi_smem_floats(dm.K);   // [128]
+  const int nck = p.f32_chunks;
+  const int tile = blockIdx.x / nck, ck = blockIdx.x % nck;
+  const int j0 = tile * kTileRows, c0 = ck * kF32Cols;
+  float* xs = fs;                                        // [128][kF32XStride]; later zs [128][E16 + 1]
+  float* zs = fs;
+  const size_t big = static_cast<size_t>(kF32Cols) * kF32XStride > 128 * static_cast<size_t>(E16 + 1)
+                         ? static_cast<size_t>(kF32Cols) * kF32XStride : 128 * static_cast<size_t>(E16 + 1);
+  float* wsm = fs + big;                                 // [E][128]
+  float* ga = wsm + E * kF32Cols;                        // [128]
+  float* gb = ga + kF32Cols;                             // [128]
+  float* hsum = gb + kF32Cols;                           // [128] second half's Gaussian sums
+  float* gcw = hsum + kF32Cols;                          // [8] per-warp constant terms
+  float* epi = gcw + 8;
+  float* dll_s = epi + epi_smem_floats(dm.K);            // [128]
+  int* flag_s = reinterpret_cast<int*>(dll_s + 128);
   uint64_t* bars = reinterpret_cast<uint64_t*>(
-      (reinterpret_cast<uintptr_t>(dll_s + 128) + 7) & ~uintptr_t(7));   // [kEpiBars]
+      (reinterpret_cast<uintptr_t>(dll_s + 3 * 128) + 7) & ~uintptr_t(7));   // [kEpiBars]
   int* abort_flag = reinterpret_cast<int*>(bars + kEpiBars);
 
-  const int t = threadIdx.x, r = t >> 2, qd = t & 3;
-  const int tile = blockIdx.x;
-  const int j0 = tile * kTileRows;
+  const int t = threadIdx.x, r = t & 127, h = t >> 7;
   pdl_wait();
   pdl_trigger();
+  const float* X = static_cast<const float*>(p.X);
+  const float* W = static_cast<const float*>(p.W);
+  // the tile's 128 x 128 block of X and the [E, 128] block of W, zero past T and d
+  for (int i = t; i < 128 * (kF32Cols / 4); i += 256) {
+    const int rr = i >> 5, q = (i & 31) * 4;
+    const bool in = j0 + rr < dm.T && c0 + q < d;
+    cp_async16(xs + rr * kF32XStride + q, in ? X + static_cast<size_t>(j0 + rr) * d + c0 + q : X, in);
+  }
+  for (int i = t; i < E * (kF32Cols / 4); i += 256) {
+    const int e = i >> 5, q = (i & 31) * 4;
+    const bool in = c0 + q < d;
+    cp_async16(wsm + e * kF32Cols + q, in ? W + static_cast<size_t>(e) * d + c0 + q : W, in);
+  }
+  asm volatile("cp.async.commit_group;" ::: "memory");
   if (t == 0) {
     *abort_flag = 0;
     init_epi_bars(bars);
     fence_mbar_init();
   }
-  float gc = 0.f;
-  if (kGauss) {
-    for (int i = t; i < dpad; i += 512) {
-      ga[i] = p.ws.gcoef[i];
-      gb[i] = p.ws.gcoef[p.ws.dcoef + i];
-    }
-    gc = gauss_gc(p.ws.gcoef, p.ws.dcoef);
+  if (kGauss && t < kF32Cols) {                          // this chunk's coefficients (eqs. 8-9)
+    const int c = c0 + t;
+    float a = 0.f, b = 0.f, cc = 0.f;
+    if (c < d && !gauss_coef_feature(p.mu[c], p.mu[d + c], p.var[c], p.var[d + c], a, b, cc))
+      atomicOr(p.ws.status, kStatusData);
+    ga[t] = a;
+    gb[t] = b;
+    cc = warp_sum(cc);
+    if ((t & 31) == 0) gcw[t >> 5] = cc;
   }
-  float acc[kF32MaxE / 4];
-#pragma unroll
-  for (int i = 0; i < kF32MaxE / 4; ++i) acc[i] = 0.f;
-  float gacc = 0.f;
-  const float* X = static_cast<const float*>(p.X);
-  const float* W = static_cast<const float*>(p.W);
+  asm volatile("cp.async.wait_all;" ::: "memory");
   __syncthreads();
-  for (int d0 = 0; d0 < d; d0 += 32) {
-    for (int i = t; i < 128 * 32; i += 512) {
-      const int rr = i >> 5, cc = i & 31;
-      xs[rr * 33 + cc] = (j0 + rr < dm.T && d0 + cc < d) ? X[static_cast<size_t>(j0 + rr) * d + d0 + cc] : 0.f;
-    }
-    for (int i = t; i < E * 32; i += 512) {
-      const int e = i >> 5, cc = i & 31;
-      wsm[e * 33 + cc] = (d0 + cc < d) ? W[static_cast<size_t>(e) * d + d0 + cc] : 0.f;
-    }
-    __syncthreads();
-#pragma unroll 4
-    for (int cc = 0; cc < 32; ++cc) {
-      const float x = xs[r * 33 + cc];
+
+  // partial logits of row r, experts e = 2i + h, over the chunk's features
+  float acc[kF32MaxE / 2];
 #pragma unroll
-      for (int i = 0; i < kF32MaxE / 4; ++i) {
-        const int e = qd + 4 * i;
-        if (e < E) acc[i] = fmaf(x, wsm[e * 33 + cc], acc[i]);
+  for (int i = 0; i < kF32MaxE / 2; ++i) acc[i] = 0.f;
+  float gs = 0.f;
+  const float* xr = xs + r * kF32XStride;
+#pragma unroll 2
+  for (int q = 0; q < kF32Cols; q += 4) {
+    const float4 x = *reinterpret_cast<const float4*>(xr + q);
+#pragma unroll
+    for (int i = 0; i < kF32MaxE / 2; ++i) {
+      const int e = 2 * i + h;
+      if (e < E) {
+        const float4 w = *reinterpret_cast<const float4*>(wsm + e * kF32Cols + q);
+        acc[i] = fmaf(x.x, w.x, fmaf(x.y, w.y, fmaf(x.z, w.z, fmaf(x.w, w.w, acc[i]))));
       }
-      if (kGauss && (cc & 3) == qd) gacc = fmaf(x, fmaf(ga[d0 + cc], x, gb[d0 + cc]), gacc);
     }
-    __syncthreads();
+    if (kGauss && (q >> 6) == h) {                        // half h of the features: sum x (ga x + gb)
+      const float4 a = *reinterpret_cast<const float4*>(ga + q);
+      const float4 b = *reinterpret_cast<const float4*>(gb + q);
+      gs = fmaf(x.x, fmaf(a.x, x.x, b.x), gs);
+      gs = fmaf(x.y, fmaf(a.y, x.y, b.y), gs);
+      gs = fmaf(x.z, fmaf(a.z, x.z, b.z), gs);
+      gs = fmaf(x.w, fmaf(a.w, x.w, b.w), gs);
+    }
   }
+  float* pz = p.f32_part + static_cast<size_t>(tile * nck + ck) * (E + 1) * 128;
 #pragma unroll
-  for (int i = 0; i < kF32MaxE / 4; ++i) {
-    const int e = qd + 4 * i;
-    if (e < E16) zs[r * (E16 + 1) + e] = (e < E) ? acc[i] : 0.f;
+  for (int i = 0; i < kF32MaxE / 2; ++i) {
+    const int e = 2 * i + h;
+    if (e < E) pz[e * 128 + r] = acc[i];
   }
-  gacc += __shfl_xor_sync(0xffffffffu, gacc, 1);
-  gacc += __shfl_xor_sync(0xffffffffu, gacc, 2);
-  if (qd == 0) dll_s[r] = gacc + gc;
+  if (kGauss) {
+    if (h == 1) hsum[r] = gs;
+    __syncthreads();
+    if (h == 0) {
+      const float gc = ((gcw[0] + gcw[1]) + (gcw[2] + gcw[3]));
+      pz[E * 128 + r] = (gs + hsum[r]) - 0.5f * gc;
+    }
+  }
+  // the last CTA of the tile sums the chunks in order and runs the epilogue
+  __threadfence();
   __syncthreads();
-  if (t < 256) {
-    const int grp = t >> 7, row = t & 127;
+  if (t == 0) *flag_s = atomicAdd(p.tile_ticket + tile, 1u) == static_cast<uint32_t>(nck - 1);
+  __syncthreads();
+  if (!*flag_s) return;
+  __threadfence();
+  if (t == 0) p.tile_ticket[tile] = 0u;                  // ready for the next call
+  const float* pt = p.f32_part + static_cast<size_t>(tile * nck) * (E + 1) * 128;
+  for (int i = 0; i < (E16 + 1) / 2 + 1; ++i) {
+    const int e = 2 * i + h;
+    if (e > E16) break;
+    float z = 0.f;
+    if (e < E || (kGauss && e == E)) {
+      for (int c = 0; c < nck; ++c) z += __ldcg(pt + static_cast<size_t>(c) * (E + 1) * 128 + e * 128 + r);
+    }
+    if (e < E16) zs[r * (E16 + 1) + e] = z;            // padding experts: logit 0, masked below
+    if (kGauss && e == E) dll_s[r] = z;
+  }
+  __syncthreads();
+  {
+    const int grp = h, row = r;
     struct Src {
       const float* z;
       int E;
@@ -1312,8 +1371,10 @@ cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s) {
     auto k = gauss ? k_router_fwd_f32<true, KM> : k_router_fwd_f32<false, KM>;
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(k, dim3(p.n_tiles), dim3(512), smem, s, p);
+    return launch_pdl(k, dim3(p.n_tiles * p.f32_chunks), dim3(256), smem, s, p);
   });
 }
+
+int f32_chunks(int d) { return (d + kF32Cols - 1) / kF32Cols; }
 
 }  // namespace smoes

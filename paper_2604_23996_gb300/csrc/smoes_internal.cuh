@@ -94,6 +94,11 @@ struct FwdParams {
   FusedPerm perm;
   int n_tiles;
   uint64_t limit_ns;
+  // fp32 path: feature chunks per tile, per-(tile, chunk) partial logits and Gaussian sums
+  // [n_tiles * f32_chunks][E + 1][128], per-tile tickets [n_tiles] (zero between calls)
+  int f32_chunks;
+  float* f32_part;
+  uint32_t* tile_ticket;
 };
 
 struct BwdParams {
@@ -166,6 +171,33 @@ struct AttnParams {
   uint64_t limit_ns;
 };
 
+// Online Gaussian statistics (eqs. 5-7): state N [2], S_mu [2, d], S_var [2, d] (fp64, updated
+// in place); per-block shifted sums part [G][4][d] and vision-row counts nvis [G] (workspace).
+struct StatsParams {
+  int T, d, G;
+  const void* X;
+  const uint8_t* is_vision;
+  double beta;
+  double* N;
+  double* S_mu;
+  double* S_var;
+  float* mu_out;             // [2, d] S_mu / N or null
+  float* var_out;            // [2, d] S_var / N or null
+  float* part;
+  int32_t* nvis;
+  double* N0;                // [2] copy of N_{t-1}
+};
+
+// Momentum-adaptive binning (eqs. 10-11).
+struct BinsParams {
+  int E, N_B;
+  double beta;
+  const int32_t* counts;     // [2, E] this step's selections by hard modality
+  double* C_bar;             // [2, E] EMA loads, updated in place
+  int32_t* expert_bin;       // [E] output
+  double* f_spec;            // [E] output or null
+};
+
 // Fixed-size scratch of smoes_bin_permute_noalloc, kept in a file-scope __device__ array of
 // bin_permute.cu (for callers that cannot allocate): room for 1024 permutation blocks x 32 bins
 // and 256 experts, which covers every plan smoes_plan_create accepts.
@@ -214,6 +246,7 @@ cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
                                    const CUtensorMap& tmW, const CUtensorMap* tmG, int n_sms,
                                    cudaStream_t s);
 cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s);
+int f32_chunks(int d);     // feature chunks of the fp32 forward and backward (128 features each)
 cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX,
                                    const CUtensorMap& tmW, const CUtensorMap& tmDX,
                                    cudaStream_t s);
@@ -225,6 +258,8 @@ cudaError_t launch_gauss_score(const GaussParams& p, smoes_dtype dt, int n_sms, 
 // Coefficients of the Gaussian log-likelihood difference (eq. 8) into coef = ga | gb | part.
 cudaError_t launch_gauss_coef(const float* mu, const float* var, int d, int dcoef, float* coef,
                               uint32_t* status, cudaStream_t s);
+cudaError_t launch_stats_update(const StatsParams& p, bool bf16, cudaStream_t s);
+cudaError_t launch_adaptive_bins(const BinsParams& p, cudaStream_t s);
 cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                              int n_sms, cudaStream_t s);
 

@@ -41,6 +41,8 @@ CASES = {
     "split_odd_chunks": (9, 650, 256, 80, 5, 5, [330, 320], torch.bfloat16, True),
     "contig_no_split": (10, 500, 192, 96, 6, 8, [250, 250], torch.bfloat16, False),
     "fp32_split": (11, 300, 96, 64, 4, 8, [150, 150], torch.float32, True),
+    # the fp32 path splits d into 128-feature chunks: three chunks, the last one partial
+    "fp32_chunks": (12, 900, 328, 48, 5, 6, [400, 500], torch.float32, True),
 }
 
 
