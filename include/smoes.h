@@ -170,10 +170,12 @@ smoes_status smoes_router_fwd(smoes_plan plan, const void* X, const void* W, con
 /* (2b) The forward (2) and the bin permutation (4) of its own top-k in one launch.
  *   Arguments: those of smoes_router_fwd, then those of smoes_bin_permute (topk_idx is the
  *   forward's output); results are identical to smoes_router_fwd followed by smoes_bin_permute.
- *   On bf16 plans the forward kernel counts each CTA's (token, bin) pairs from the top-k it holds
- *   in registers; after a grid-wide barrier (a cooperative launch: every CTA resident) the warps
- *   that are idle once the CTA's gate GEMM is done place the CTA's entries, while the per-sample
- *   MI reduction of eqs. (12)-(15) runs. fp32 plans make the two calls. The paper has no
+ *   On bf16 plans with at most two 128-token tiles per SM the forward kernel counts each CTA's
+ *   (token, bin) pairs from the top-k it holds in registers; after a grid-wide barrier (a
+ *   cooperative launch: every CTA resident) the warps that are idle once the CTA's gate GEMM is
+ *   done place the CTA's entries, while the per-sample MI reduction of eqs. (12)-(15) runs.
+ *   Larger batches and fp32 plans make the two calls (the fused scatter runs after a CTA's last
+ *   tile, serially over its tokens, and loses to the standalone kernel there). The paper has no
  *   counterpart for this fusion; it removes the separate launch and counting pass. */
 smoes_status smoes_router_fwd_permute(smoes_plan plan, const void* X, const void* W,
                                       const float* M_in, const smoes_gauss_args* gauss,

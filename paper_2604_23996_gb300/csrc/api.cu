@@ -504,8 +504,13 @@ smoes_status smoes_router_fwd_permute(smoes_plan P, const void* X, const void* W
   if (!bin_offsets || !dispatch) return SMOES_ERR_INVALID_ARG;
   if (expert_counts && !is_vision) return SMOES_ERR_INVALID_ARG;
   if (d.T > 0 && (!perm_token || !perm_mask)) return SMOES_ERR_INVALID_ARG;
-  // inside the forward launch on the tensor-core path; otherwise the two calls in order
-  if (d.dtype == SMOES_BF16 && d.T > 0 && d.n_bins <= kMaxBins && d.E <= kMaxExperts) {
+  // inside the forward launch on the tensor-core path when every CTA holds at most two tiles
+  // (the fused scatter runs after a CTA's last tile, serially over its tokens: with many tiles
+  // per CTA the standalone permutation, spread over the whole GPU, is faster); otherwise the two
+  // calls in order
+  const int fwd_tiles = (d.T + kFwdBM - 1) / kFwdBM;
+  if (d.dtype == SMOES_BF16 && d.T > 0 && d.n_bins <= kMaxBins && d.E <= kMaxExperts &&
+      fwd_tiles <= 2 * P->n_sms) {
     FusedPerm f{};
     f.home = home;
     f.is_vision = is_vision;

@@ -69,8 +69,9 @@ __global__ void __launch_bounds__(kPermThreads) k_perm(const PermParams p) {
   __shared__ int disp[kMaxBins * kMaxBins];
   __shared__ int ecnt[2 * kMaxExperts];
   __shared__ int ok_s;
-  // launched without programmatic serialization (a cooperative grid): everything before it has
-  // completed, so the next kernel may be scheduled now
+  // a cooperative grid launched with programmatic serialization: the top-k of the kernel before
+  // it are read only after that kernel has completed
+  pdl_wait();
   pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int K = p.K;
@@ -324,11 +325,13 @@ cudaError_t launch_bin_permute(const PermParams& p, cudaStream_t s) {
   cfg.gridDim = dim3(p.n_blocks);
   cfg.blockDim = dim3(kPermThreads);
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeCooperative;    // every block resident: the barrier is safe
   attr[0].val.cooperative = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return with_kernel(p.k, [&](auto kern) { return cudaLaunchKernelEx(&cfg, kern, p); });
 }
 

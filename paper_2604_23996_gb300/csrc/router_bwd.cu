@@ -89,96 +89,126 @@ __device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
 // ~2^-17 relative) in the 128-byte-swizzled operand image of its 64-token tile,
 // [tile][hi | lo][E_pad/64][64 rows][128 B], which the main kernel bulk-copies. Rows beyond T and
 // padded experts are zeros. With consecutive bins of a multiple of 4 experts, a thread's 8
-// experts lie in at most two bins: their coefficients are read once per bin.
-template <int TPT>
+// experts lie in at most two bins: their coefficients are read once per bin. Every thread group
+// handles kDzRep tokens (a block's token sets kDzRep apart) with all their loads issued before
+// any is used, so enough bytes are in flight to stream the saved scores at HBM speed. kUp: an
+// upstream gradient of the top-k weights is present (its per-token tables stay out of the
+// register budget otherwise).
+constexpr int kDzRep = 2;
+
+template <int TPT, bool kUp>
 __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
   pdl_wait();                                         // scores and tables of the forward
   pdl_trigger();
   const Dims& dm = p.dm;
   const int E = dm.E, K = dm.K, k = dm.k;
   constexpr int kEp = TPT * 8;
-  const int j = (blockIdx.x * 256 + threadIdx.x) / TPT;
+  constexpr int kGroups = 256 / TPT;                  // token groups per block and set
   const int c = threadIdx.x % TPT;
   const int e0 = c * 8;
   const int n_rows = p.n_tiles * kBwdBT;
-  if (j >= n_rows) return;                            // whole TPT groups exit together
-  const bool valid = j < dm.T;
-  float g[8], u[8];
-  if (valid) {
-    const float* grow = p.ws.gsave + static_cast<size_t>(j) * E;
-    const float ginv = __ldcg(p.ws.ginv + j);
-    if ((E & 3) == 0 && e0 + 8 <= E) {
-      const float4 a = __ldcg(reinterpret_cast<const float4*>(grow + e0));
-      const float4 b = __ldcg(reinterpret_cast<const float4*>(grow + e0 + 4));
-      g[0] = a.x; g[1] = a.y; g[2] = a.z; g[3] = a.w; g[4] = b.x; g[5] = b.y; g[6] = b.z; g[7] = b.w;
-    } else {
+  int j[kDzRep];
+  bool valid[kDzRep];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) g[q] = (e0 + q < E) ? __ldcg(grow + e0 + q) : 0.f;
+  for (int q = 0; q < kDzRep; ++q) {
+    j[q] = (blockIdx.x * kDzRep + q) * kGroups + threadIdx.x / TPT;
+    valid[q] = j[q] < dm.T;
+  }
+  // every load of the block's tokens first
+  float4 ga[kDzRep], gb[kDzRep];
+  float ginv[kDzRep];
+  float2 m[kDzRep];
+  int smp[kDzRep];
+  const bool vec = (E & 3) == 0 && e0 + 8 <= E;
+#pragma unroll
+  for (int q = 0; q < kDzRep; ++q) {
+    ga[q] = gb[q] = make_float4(0.f, 0.f, 0.f, 0.f);
+    ginv[q] = 0.f;
+    m[q] = make_float2(0.5f, 0.5f);
+    smp[q] = 0;
+    if (valid[q]) {
+      const float* grow = p.ws.gsave + static_cast<size_t>(j[q]) * E;
+      if (vec) {
+        ga[q] = __ldcg(reinterpret_cast<const float4*>(grow + e0));
+        gb[q] = __ldcg(reinterpret_cast<const float4*>(grow + e0 + 4));
+      } else {
+        float t[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) t[u] = (e0 + u < E) ? __ldcg(grow + e0 + u) : 0.f;
+        ga[q] = make_float4(t[0], t[1], t[2], t[3]);
+        gb[q] = make_float4(t[4], t[5], t[6], t[7]);
+      }
+      ginv[q] = __ldcg(p.ws.ginv + j[q]);
+      m[q] = __ldg(reinterpret_cast<const float2*>(p.M) + j[q]);
+      smp[q] = __ldg(p.ws.token_sample + j[q]);
     }
+  }
 #pragma unroll
-    for (int q = 0; q < 8; ++q) g[q] *= ginv;                 // the softmax score g_je
-    const float2 m = __ldg(reinterpret_cast<const float2*>(p.M) + j);
-    const float dv = m.x - 0.5f, dt = m.y - 0.5f;
-    // the sample's coefficient table was written by the forward kernel and is read-only here
-    const float* tb = p.ws.tabs + static_cast<size_t>(__ldg(p.ws.token_sample + j)) * 3 * K;
-    if (dm.contig_bins && e0 + 8 <= E) {
-      const int b0 = e0 / dm.N_B, b1 = (e0 + 7) / dm.N_B;
-      const float u0 = __ldg(tb + 2 * K + b0) + dv * __ldg(tb + b0) + dt * __ldg(tb + K + b0);
-      const float u1 = __ldg(tb + 2 * K + b1) + dv * __ldg(tb + b1) + dt * __ldg(tb + K + b1);
+  for (int q = 0; q < kDzRep; ++q) {
+    if (j[q] >= n_rows) continue;                     // whole TPT groups skip together
+    float g[8] = {ga[q].x, ga[q].y, ga[q].z, ga[q].w, gb[q].x, gb[q].y, gb[q].z, gb[q].w};
+    float u[8];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) u[q] = (e0 + q) / dm.N_B == b0 ? u0 : u1;
-    } else {
+    for (int i = 0; i < 8; ++i) { g[i] *= ginv[q]; u[i] = 0.f; }        // the softmax score g_je
+    if (valid[q]) {
+      const float dv = m[q].x - 0.5f, dt = m[q].y - 0.5f;
+      // the sample's coefficient table was written by the forward kernel and is read-only here
+      const float* tb = p.ws.tabs + static_cast<size_t>(smp[q]) * 3 * K;
+      if (dm.contig_bins && e0 + 8 <= E) {
+        const int b0 = e0 / dm.N_B, b1 = (e0 + 7) / dm.N_B;
+        const float u0 = __ldg(tb + 2 * K + b0) + dv * __ldg(tb + b0) + dt * __ldg(tb + K + b0);
+        const float u1 = __ldg(tb + 2 * K + b1) + dv * __ldg(tb + b1) + dt * __ldg(tb + K + b1);
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        u[q] = 0.f;
-        if (e0 + q < E) {
-          const int b = __ldg(p.ws.expert_bin + e0 + q);
-          u[q] = __ldg(tb + 2 * K + b) + dv * __ldg(tb + b) + dt * __ldg(tb + K + b);
+        for (int i = 0; i < 8; ++i) u[i] = (e0 + i) / dm.N_B == b0 ? u0 : u1;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          if (e0 + i < E) {
+            const int b = __ldg(p.ws.expert_bin + e0 + i);
+            u[i] = __ldg(tb + 2 * K + b) + dv * __ldg(tb + b) + dt * __ldg(tb + K + b);
+          }
         }
       }
     }
-  } else {
+    float part = 0.f;
 #pragma unroll
-    for (int q = 0; q < 8; ++q) { g[q] = 0.f; u[q] = 0.f; }
-  }
-  float part = 0.f;
+    for (int i = 0; i < 8; ++i) part = fmaf(g[i], u[i], part);
 #pragma unroll
-  for (int q = 0; q < 8; ++q) part = fmaf(g[q], u[q], part);
+    for (int o = 1; o < TPT; o <<= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+    float dz[8];
 #pragma unroll
-  for (int o = 1; o < TPT; o <<= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-  float dz[8];
+    for (int i = 0; i < 8; ++i) dz[i] = p.scale * g[i] * (u[i] - part);
+    if (kUp && valid[q]) {
+      Upstream up;
+      load_upstream(p, j[q], up);
 #pragma unroll
-  for (int q = 0; q < 8; ++q) dz[q] = p.scale * g[q] * (u[q] - part);
-  if (valid && p.d_topk_w != nullptr) {
-    Upstream up;
-    load_upstream(p, j, up);
-#pragma unroll
-    for (int q = 0; q < 8; ++q)
-      if (e0 + q < E) dz[q] += g[q] * (upstream_at(up, k, e0 + q) - up.gdt);
-  }
-  if (valid && p.dlogits) {
-    float* dl = p.dlogits + static_cast<size_t>(j) * E;
-    if ((E & 3) == 0 && e0 + 8 <= E) {
-      *reinterpret_cast<float4*>(dl + e0) = make_float4(dz[0], dz[1], dz[2], dz[3]);
-      *reinterpret_cast<float4*>(dl + e0 + 4) = make_float4(dz[4], dz[5], dz[6], dz[7]);
-    } else {
-#pragma unroll
-      for (int q = 0; q < 8; ++q)
-        if (e0 + q < E) dl[e0 + q] = dz[q];
+      for (int i = 0; i < 8; ++i)
+        if (e0 + i < E) dz[i] += g[i] * (upstream_at(up, k, e0 + i) - up.gdt);
     }
-  }
-  uint32_t hw[4], lw[4];
+    if (valid[q] && p.dlogits) {
+      float* dl = p.dlogits + static_cast<size_t>(j[q]) * E;
+      if (vec) {
+        *reinterpret_cast<float4*>(dl + e0) = make_float4(dz[0], dz[1], dz[2], dz[3]);
+        *reinterpret_cast<float4*>(dl + e0 + 4) = make_float4(dz[4], dz[5], dz[6], dz[7]);
+      } else {
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    const __nv_bfloat16 h0 = __float2bfloat16_rn(dz[2 * q]), h1 = __float2bfloat16_rn(dz[2 * q + 1]);
-    hw[q] = static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
-    lw[q] = pack_bf16x2(dz[2 * q] - __bfloat162float(h0), dz[2 * q + 1] - __bfloat162float(h1));
+        for (int i = 0; i < 8; ++i)
+          if (e0 + i < E) dl[e0 + i] = dz[i];
+      }
+    }
+    uint32_t hw[4], lw[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat16 h0 = __float2bfloat16_rn(dz[2 * i]), h1 = __float2bfloat16_rn(dz[2 * i + 1]);
+      hw[i] = static_cast<uint32_t>(__bfloat16_as_ushort(h0)) | (static_cast<uint32_t>(__bfloat16_as_ushort(h1)) << 16);
+      lw[i] = pack_bf16x2(dz[2 * i] - __bfloat162float(h0), dz[2 * i + 1] - __bfloat162float(h1));
+    }
+    const int tile = j[q] / kBwdBT, r = j[q] % kBwdBT;
+    uint8_t* img = p.ws.dz_img + static_cast<size_t>(tile) * (2 * kEp * 128);
+    const uint32_t off = (e0 >> 6) * 8192u + sw128_offset(static_cast<uint32_t>(r), static_cast<uint32_t>(e0 & 63));
+    *reinterpret_cast<uint4*>(img + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    *reinterpret_cast<uint4*>(img + kEp * 128 + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
   }
-  const int tile = j / kBwdBT, r = j % kBwdBT;
-  uint8_t* img = p.ws.dz_img + static_cast<size_t>(tile) * (2 * kEp * 128);
-  const uint32_t off = (e0 >> 6) * 8192u + sw128_offset(static_cast<uint32_t>(r), static_cast<uint32_t>(e0 & 63));
-  *reinterpret_cast<uint4*>(img + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-  *reinterpret_cast<uint4*>(img + kEp * 128 + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
 }
 
 // ------------------------------------------------------------------ tcgen05 backward (bf16)
@@ -187,22 +217,32 @@ struct BwdLayout {
   uint32_t wsl, dz, xst, stg, bars, total;
 };
 
+// dX^T accumulators in TMEM: kDxBufs buffers of 64 columns after the dW^T blocks (which take at
+// most 256 columns: slice width x E_pad = 32768), drained by two warp groups in turn.
+constexpr int kDxBufs = 4;
+constexpr int kDrainGroups = 2;
+constexpr int kBwdThreads = 64 + kDrainGroups * 128;
+
 __host__ __device__ inline BwdLayout bwd_layout(int E_pad, int n_xst) {
   BwdLayout L;
   uint32_t o = 0;
   L.wsl = o;  o += 65536u;                                         // W slice (ds * E_pad * 2 B)
   L.dz = o;   o += 2u * 2u * static_cast<uint32_t>(E_pad) * 128u;   // 2 buffers x (hi, lo)
   L.xst = o;  o += static_cast<uint32_t>(n_xst) * 16384u;          // X stages [2 atoms][64][128 B]
-  L.stg = o;  o += 2u * 16384u;                                    // dX staging [64][128] bf16 x2
-  L.bars = o; o += 8u * (2u * n_xst + 18u) + 16u;
+  L.stg = o;  o += kDrainGroups * 16384u;                          // dX staging [64][128] bf16 per group
+  L.bars = o; o += 8u * (2u * n_xst + 32u) + 16u;
   L.total = o + 1024u;
   return L;
 }
 
-// Roles (192 threads): warp 0 TMA / bulk-copy producer, warp 1 MMA issuer, warps 2-5 dX drain
-// and dW^T drain. After the last tile every CTA writes its dW^T partial; k_dw_reduce sums them.
+// Roles (320 threads): warp 0 TMA / bulk-copy producer, warp 1 MMA issuer, warps 2-5 and 6-9 two
+// drain groups: d-block iteration `it` of the CTA uses dX^T buffer it % 4 and is drained by group
+// it % 2 through the group's own staging buffer, so two drains run while the tensor cores fill
+// the other buffers. An X stage is released as soon as the d-block's dW^T MMAs complete (the dX^T
+// MMAs read W and dz only). After the last tile every CTA writes its dW^T partial (both groups,
+// alternate d-blocks); k_dw_reduce sums them.
 template <int E_pad>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(kBwdThreads, 1)
 k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
                 const __grid_constant__ CUtensorMap tmDX, const BwdParams p, const int n_xst) {
   extern __shared__ uint8_t smem_raw[];
@@ -218,14 +258,14 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   uint64_t* xempty = bars + n_xst;
   uint64_t* dz_full = bars + 2 * n_xst;       // [2] the tile's dz image has landed
   uint64_t* dz_empty = dz_full + 2;           // [2] the tile's MMAs have read it
-  uint64_t* dx_full = dz_full + 4;            // [2]
-  uint64_t* dx_empty = dz_full + 6;           // [2]
-  uint64_t* wfull = dz_full + 8;
-  uint64_t* dw_full = dz_full + 9;
-  uint64_t* drain = dz_full + 10;
-  uint64_t* stg_free = dz_full + 11;          // [2] staging buffer may be rewritten
-  uint64_t* stg_full = dz_full + 13;          // [2] staging buffer written
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(dz_full + 18);
+  uint64_t* dx_full = dz_full + 4;            // [kDxBufs]
+  uint64_t* dx_empty = dx_full + kDxBufs;     // [kDxBufs]
+  uint64_t* wfull = dx_empty + kDxBufs;
+  uint64_t* dw_full = wfull + 1;
+  uint64_t* drain = wfull + 2;
+  uint64_t* stg_free = wfull + 3;             // [kDrainGroups] a group's staging may be rewritten
+  uint64_t* stg_full = stg_free + kDrainGroups;   // [kDrainGroups] a group's staging is written
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(stg_full + kDrainGroups);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -247,8 +287,12 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     for (int i = 0; i < 2; ++i) {
       mbar_init(dz_full + i, 1);
       mbar_init(dz_empty + i, 1);
+    }
+    for (int i = 0; i < kDxBufs; ++i) {
       mbar_init(dx_full + i, 1);
       mbar_init(dx_empty + i, 128);
+    }
+    for (int i = 0; i < kDrainGroups; ++i) {
       mbar_init(stg_free + i, 1);
       mbar_init(stg_full + i, 128);
     }
@@ -265,7 +309,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tm_dx = tmem + 256u;          // two 64-column dX^T buffers after the dW^T blocks
+  const uint32_t tm_dx = tmem + 256u;          // kDxBufs 64-column dX^T buffers after the dW^T blocks
   if (warp == 0 && lane == 0) {
     // W slice (atom a = columns d0 + 64a .. +64), requested before the dz prep kernel has
     // finished: that kernel does not write W, and it started only after all earlier work
@@ -319,8 +363,9 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       const uint32_t id_dx = idesc_bf16(128, kBwdBT, true, false);
       bool ok = mbar_wait(wfull, 0, wc);
       tc_fence_after();
-      int st = 0, xb = 0;
-      uint32_t ph = 0, xph = 0;
+      int st = 0;
+      uint32_t ph = 0;
+      int it = 0;                              // d-block iterations of this CTA
       int lt = 0;
       for (int t = grp; t < p.n_tiles && ok; t += G, ++lt) {
         const int zb = lt & 1;
@@ -329,7 +374,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
         tc_fence_after();
         const uint32_t hi = smem_u32(dzb + zb * dz_buf_bytes);
         const uint32_t lo = hi + dz_half;
-        for (int b = 0; b < nb; ++b) {
+        for (int b = 0; b < nb; ++b, ++it) {
           if (!mbar_wait(xfull + st, ph, wc)) { ok = false; break; }
           tc_fence_after();
           const uint32_t xs = smem_u32(xst + st * 16384);
@@ -342,8 +387,12 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
             umma_bf16(dwc, da, dh, id_dw, (lt > 0 || ks > 0) ? 1u : 0u);
             umma_bf16(dwc, da, dl, id_dw, 1u);
           }
+          umma_commit(xempty + st);             // the X stage is free once these MMAs complete
+          if (++st == n_xst) { st = 0; ph ^= 1u; }
           if (want_dx) {
-            if (!mbar_wait(dx_empty + xb, xph ^ 1u, wc)) { ok = false; break; }
+            const int xb = it % kDxBufs;
+            const uint32_t xuse = static_cast<uint32_t>(it / kDxBufs);
+            if (!mbar_wait(dx_empty + xb, (xuse & 1u) ^ 1u, wc)) { ok = false; break; }
             tc_fence_after();
             const uint32_t dxc = tm_dx + static_cast<uint32_t>(xb * kBwdBT);
             const uint32_t wa = smem_u32(wsl + 2 * b * dz_half);
@@ -357,10 +406,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
               umma_bf16(dxc, da, dl, id_dx, 1u);
             }
             umma_commit(dx_full + xb);
-            if (++xb == 2) { xb = 0; xph ^= 1u; }
           }
-          umma_commit(xempty + st);
-          if (++st == n_xst) { st = 0; ph ^= 1u; }
         }
         if (!ok) break;
         umma_commit(dz_empty + zb);
@@ -373,27 +419,28 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
       mbar_wait(drain, 0, wd);
     }
   } else {
-    // -------------------------------------------------------------- dX epilogue + dW drain
-    const int lg = warp & 3;
-    const int etid = threadIdx.x - 64;                 // 0..127
-    const bool issuer = (etid == 0);
-    int xb = 0;
-    uint32_t xph = 0;
-    int it = 0;
+    // -------------------------------------------------------------- dX drain + dW drain (2 groups)
+    const int lg = warp & 3;                           // TMEM lane quarter of this warp
+    const int dg = (warp - 2) >> 2;                    // drain group
+    const int gtid = (threadIdx.x - 64) & 127;         // 0..127 within the group
+    const bool issuer = (gtid == 0);
+    uint8_t* sgb = stg + dg * 16384;
     bool ok = true;
     if (want_dx) {
+      int it = 0, n_mine = 0;
       for (int t = grp; t < p.n_tiles && ok; t += G) {
         for (int b = 0; b < nb; ++b, ++it) {
-          if (!mbar_wait(dx_full + xb, xph, wc)) { ok = false; break; }
+          if ((it & 1) != dg) continue;
+          const int xb = it % kDxBufs;
+          const uint32_t xuse = static_cast<uint32_t>(it / kDxBufs);
+          if (!mbar_wait(dx_full + xb, xuse & 1u, wc)) { ok = false; break; }
           tc_fence_after();
-          const int sb = it & 1;
-          const uint32_t suse = static_cast<uint32_t>(it >> 1);
-          if (issuer) {                                // staging[sb] free again
-            tma_store_wait_read<1>();
-            mbar_arrive(stg_free + sb);
+          if (issuer) {                                // this group's staging free again
+            tma_store_wait_read<0>();
+            mbar_arrive(stg_free + dg);
           }
-          if (!mbar_wait(stg_free + sb, suse & 1u, wc)) { ok = false; break; }
-          __nv_bfloat16* sg = reinterpret_cast<__nv_bfloat16*>(stg + sb * 16384);
+          if (!mbar_wait(stg_free + dg, static_cast<uint32_t>(n_mine & 1), wc)) { ok = false; break; }
+          __nv_bfloat16* sg = reinterpret_cast<__nv_bfloat16*>(sgb);
           const uint32_t ta = tm_dx + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(xb * kBwdBT);
           const int drow = lg * 32 + lane;
 #pragma unroll
@@ -405,25 +452,26 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
           }
           tc_fence_before();
           mbar_arrive(dx_empty + xb);
-          if (++xb == 2) { xb = 0; xph ^= 1u; }
           fence_proxy_async_smem();
-          mbar_arrive(stg_full + sb);
+          mbar_arrive(stg_full + dg);
           if (issuer) {
-            if (!mbar_wait(stg_full + sb, suse & 1u, wc)) { ok = false; break; }
+            if (!mbar_wait(stg_full + dg, static_cast<uint32_t>(n_mine & 1), wc)) { ok = false; break; }
             tma_store_2d(&tmDX, sg, d0 + b * kBwdBD, t * kBwdBT);
             tma_store_commit();
           }
+          ++n_mine;
         }
       }
       if (issuer) tma_store_wait_all<0>();
     }
-    // partial dW^T of this group: lanes = d rows, columns = experts
+    // partial dW^T of this group: lanes = d rows, columns = experts; the two drain groups take
+    // alternate d-blocks
     if (ok && mbar_wait(dw_full, 0, wc)) {
       tc_fence_after();
-      for (int b = 0; b < nb; ++b) {
+      for (int b = dg; b < nb; b += kDrainGroups) {
         const int drow = d0 + b * kBwdBD + lg * 32 + lane;
         const uint32_t ta = tmem + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>(b * E_pad);
-#pragma unroll
+#pragma unroll 1
         for (int c = 0; c < E_pad / 32; ++c) {
           float v[32];
           tmem_ld32(ta + 32u * c, v);
@@ -453,6 +501,8 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
 constexpr int kF32MaxE = 64;
 constexpr int kF32Cols = 128;
 
+// EB = E rounded up to 16: the expert loops run to EB over zero-padded dz and W columns.
+template <int EB>
 __global__ void __launch_bounds__(256)
 k_router_bwd_f32(const BwdParams p) {
   extern __shared__ float bs[];
@@ -462,8 +512,9 @@ k_router_bwd_f32(const BwdParams p) {
   const int E = dm.E, K = dm.K, k = dm.k;
   const int nck = (dm.d + kF32Cols - 1) / kF32Cols;
   const int tile = blockIdx.x / nck, ck = blockIdx.x % nck;
-  float* dzs = bs;                                   // [64][E+1]
-  float* dws = dzs + 64 * (E + 1);                   // [E][128] second half's dW partial
+  constexpr int kZs = EB + 4;                        // dz row stride (16-byte aligned rows)
+  float* dzs = bs;                                   // [64][kZs], experts past E zero
+  float* dws = dzs + 64 * kZs;                       // [E][128] second half's dW partial
   const int t = threadIdx.x;
   {
     const int r = t >> 2, qd = t & 3;
@@ -491,9 +542,9 @@ k_router_bwd_f32(const BwdParams p) {
     }
     part += __shfl_xor_sync(0xffffffffu, part, 1);
     part += __shfl_xor_sync(0xffffffffu, part, 2);
-    for (int e = qd; e < E; e += 4) {
+    for (int e = qd; e < EB; e += 4) {
       float v = 0.f;
-      if (valid) {
+      if (valid && e < E) {
         const int b = p.ws.expert_bin[e];
         const float u = tb[2 * K + b] + dv * tb[b] + dt * tb[K + b];
         const float ge = g[e] * ginv;
@@ -501,7 +552,7 @@ k_router_bwd_f32(const BwdParams p) {
         if (has_up) v += ge * (upstream_at(up, k, e) - up.gdt);
         if (p.dlogits && ck == 0) p.dlogits[static_cast<size_t>(j) * E + e] = v;
       }
-      dzs[r * (E + 1) + e] = v;
+      dzs[r * kZs + e] = v;
     }
   }
   const float* X = static_cast<const float*>(p.X);
@@ -509,9 +560,9 @@ k_router_bwd_f32(const BwdParams p) {
   float* dX = static_cast<float*>(p.dX);
   const int c = ck * kF32Cols + (t & 127), h = t >> 7;
   const bool cin = c < dm.d;
-  float wc[kF32MaxE], acc[kF32MaxE];
+  float wc[EB], acc[EB];
 #pragma unroll
-  for (int e = 0; e < kF32MaxE; ++e) {
+  for (int e = 0; e < EB; ++e) {
     wc[e] = (e < E && cin) ? __ldg(W + static_cast<size_t>(e) * dm.d + c) : 0.f;
     acc[e] = 0.f;
   }
@@ -529,15 +580,16 @@ k_router_bwd_f32(const BwdParams p) {
 #pragma unroll
     for (int u = 0; u < kU; ++u) {
       if (rb + u >= rows) break;
-      const float* zr = dzs + (r0 + rb + u) * (E + 1);
+      const float* zr = dzs + (r0 + rb + u) * kZs;
       float dx = 0.f;
 #pragma unroll
-      for (int e = 0; e < kF32MaxE; ++e) {
-        if (e < E) {
-          const float z = zr[e];
-          dx = fmaf(z, wc[e], dx);
-          acc[e] = fmaf(z, x[u], acc[e]);
-        }
+      for (int e = 0; e < EB; e += 4) {
+        const float4 z = *reinterpret_cast<const float4*>(zr + e);
+        dx = fmaf(z.x, wc[e], fmaf(z.y, wc[e + 1], fmaf(z.z, wc[e + 2], fmaf(z.w, wc[e + 3], dx))));
+        acc[e] = fmaf(z.x, x[u], acc[e]);
+        acc[e + 1] = fmaf(z.y, x[u], acc[e + 1]);
+        acc[e + 2] = fmaf(z.z, x[u], acc[e + 2]);
+        acc[e + 3] = fmaf(z.w, x[u], acc[e + 3]);
       }
       const size_t j = static_cast<size_t>(tile) * 64 + r0 + rb + u;
       if (dX && cin) dX[j * dm.d + c] = dx;
@@ -545,13 +597,13 @@ k_router_bwd_f32(const BwdParams p) {
   }
   if (h == 1) {
 #pragma unroll
-    for (int e = 0; e < kF32MaxE; ++e)
+    for (int e = 0; e < EB; ++e)
       if (e < E) dws[e * kF32Cols + (t & 127)] = acc[e];
   }
   __syncthreads();
   if (h == 0 && cin) {
 #pragma unroll
-    for (int e = 0; e < kF32MaxE; ++e)
+    for (int e = 0; e < EB; ++e)
       if (e < E)
         p.ws.dw_part[(static_cast<size_t>(tile) * E + e) * dm.d + c] = acc[e] + dws[e * kF32Cols + t];
   }
@@ -623,10 +675,16 @@ __global__ void __launch_bounds__(kDwSlices * kDwCols) k_dw_reduce(const BwdPara
 
 cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s) {
   const int E_pad = round_up(p.dm.E, 64);
-  const long threads = static_cast<long>(p.n_tiles) * kBwdBT * (E_pad / 8);
-  const int blocks = static_cast<int>((threads + 255) / 256);
-  if (E_pad == 64) return launch_pdl(k_dz_prep<8>, dim3(blocks), dim3(256), 0, s, p);
-  if (E_pad == 128) return launch_pdl(k_dz_prep<16>, dim3(blocks), dim3(256), 0, s, p);
+  const int tokens_per_block = kDzRep * 256 / (E_pad / 8);
+  const long rows = static_cast<long>(p.n_tiles) * kBwdBT;
+  const int blocks = static_cast<int>((rows + tokens_per_block - 1) / tokens_per_block);
+  const bool up = p.d_topk_w != nullptr;
+  if (E_pad == 64)
+    return up ? launch_pdl(k_dz_prep<8, true>, dim3(blocks), dim3(256), 0, s, p)
+              : launch_pdl(k_dz_prep<8, false>, dim3(blocks), dim3(256), 0, s, p);
+  if (E_pad == 128)
+    return up ? launch_pdl(k_dz_prep<16, true>, dim3(blocks), dim3(256), 0, s, p)
+              : launch_pdl(k_dz_prep<16, false>, dim3(blocks), dim3(256), 0, s, p);
   return cudaErrorInvalidValue;
 }
 
@@ -641,18 +699,21 @@ cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX, c
   auto k = (E_pad == 64) ? k_router_bwd_tc<64> : k_router_bwd_tc<128>;
   cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  return launch_pdl(k, dim3(p.groups * p.slices), dim3(192), smem, s, tmX, tmW, tmDX, p, n_xst);
+  return launch_pdl(k, dim3(p.groups * p.slices), dim3(kBwdThreads), smem, s, tmX, tmW, tmDX, p, n_xst);
 }
 
 
 cudaError_t launch_router_bwd_f32(const BwdParams& p, cudaStream_t s) {
   if (p.dm.E > kF32MaxE) return cudaErrorInvalidValue;
-  const size_t smem = sizeof(float) * (64 * (p.dm.E + 1) + static_cast<size_t>(p.dm.E) * kF32Cols);
-  cudaError_t e = cudaFuncSetAttribute(k_router_bwd_f32, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  const int eb = round_up(p.dm.E, 16);
+  const size_t smem = sizeof(float) * (64 * static_cast<size_t>(eb + 4) + static_cast<size_t>(p.dm.E) * kF32Cols);
+  auto k = eb <= 16 ? k_router_bwd_f32<16> : eb <= 32 ? k_router_bwd_f32<32>
+         : eb <= 48 ? k_router_bwd_f32<48> : k_router_bwd_f32<64>;
+  cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   const int nck = (p.dm.d + kF32Cols - 1) / kF32Cols;
-  return launch_pdl(k_router_bwd_f32, dim3(p.n_tiles * nck), dim3(256), smem, s, p);
+  return launch_pdl(k, dim3(p.n_tiles * nck), dim3(256), smem, s, p);
 }
 
 cudaError_t launch_dw_reduce(const BwdParams& p, cudaStream_t s) {

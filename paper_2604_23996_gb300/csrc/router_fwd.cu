@@ -1153,7 +1153,7 @@ __host__ __device__ inline size_t f32_smem_floats(const Dims& dm) {
   const int E16 = round_up(dm.E, 16);
   const size_t xs = static_cast<size_t>(kF32Cols) * kF32XStride;
   const size_t zs = 128 * static_cast<size_t>(E16 + 1);
-  return (xs > zs ? xs : zs) + static_cast<size_t>(dm.E) * kF32Cols + 3 * kF32Cols + 8 +
+  return (xs > zs ? xs : zs) + static_cast<size_t>(round_up(dm.E, 16)) * kF32Cols + 3 * kF32Cols + 8 +
          epi_smem_floats(dm.K) + 3 * 128 + 8;
 }
 
@@ -1162,7 +1162,9 @@ __device__ __forceinline__ void cp_async16(void* dst, const void* src, bool in) 
                ::"r"(smem_u32(dst)), "l"(src), "r"(in ? 16 : 0) : "memory");
 }
 
-template <bool kGauss, int KM>
+// EB = E rounded up to 16 (16, 32, 48 or 64): the expert loops are unrolled to EB with the padding
+// experts' W rows zero, so no expert is predicated off.
+template <bool kGauss, int KM, int EB>
 __global__ void __launch_bounds__(256)
 k_router_fwd_f32(const FwdParams p) {
   extern __shared__ float fs[];
@@ -1176,8 +1178,8 @@ k_router_fwd_f32(const FwdParams p) {
   float* zs = fs;
   const size_t big = static_cast<size_t>(kF32Cols) * kF32XStride > 128 * static_cast<size_t>(E16 + 1)
                          ? static_cast<size_t>(kF32Cols) * kF32XStride : 128 * static_cast<size_t>(E16 + 1);
-  float* wsm = fs + big;                                 // [E][128]
-  float* ga = wsm + E * kF32Cols;                        // [128]
+  float* wsm = fs + big;                                 // [EB][128], rows past E zero
+  float* ga = wsm + EB * kF32Cols;                       // [128]
   float* gb = ga + kF32Cols;                             // [128]
   float* hsum = gb + kF32Cols;                           // [128] second half's Gaussian sums
   float* gcw = hsum + kF32Cols;                          // [8] per-warp constant terms
@@ -1199,9 +1201,9 @@ k_router_fwd_f32(const FwdParams p) {
     const bool in = j0 + rr < dm.T && c0 + q < d;
     cp_async16(xs + rr * kF32XStride + q, in ? X + static_cast<size_t>(j0 + rr) * d + c0 + q : X, in);
   }
-  for (int i = t; i < E * (kF32Cols / 4); i += 256) {
+  for (int i = t; i < EB * (kF32Cols / 4); i += 256) {
     const int e = i >> 5, q = (i & 31) * 4;
-    const bool in = c0 + q < d;
+    const bool in = e < E && c0 + q < d;
     cp_async16(wsm + e * kF32Cols + q, in ? W + static_cast<size_t>(e) * d + c0 + q : W, in);
   }
   asm volatile("cp.async.commit_group;" ::: "memory");
@@ -1224,21 +1226,18 @@ k_router_fwd_f32(const FwdParams p) {
   __syncthreads();
 
   // partial logits of row r, experts e = 2i + h, over the chunk's features
-  float acc[kF32MaxE / 2];
+  float acc[EB / 2];
 #pragma unroll
-  for (int i = 0; i < kF32MaxE / 2; ++i) acc[i] = 0.f;
+  for (int i = 0; i < EB / 2; ++i) acc[i] = 0.f;
   float gs = 0.f;
   const float* xr = xs + r * kF32XStride;
-#pragma unroll 2
+#pragma unroll 1
   for (int q = 0; q < kF32Cols; q += 4) {
     const float4 x = *reinterpret_cast<const float4*>(xr + q);
 #pragma unroll
-    for (int i = 0; i < kF32MaxE / 2; ++i) {
-      const int e = 2 * i + h;
-      if (e < E) {
-        const float4 w = *reinterpret_cast<const float4*>(wsm + e * kF32Cols + q);
-        acc[i] = fmaf(x.x, w.x, fmaf(x.y, w.y, fmaf(x.z, w.z, fmaf(x.w, w.w, acc[i]))));
-      }
+    for (int i = 0; i < EB / 2; ++i) {
+      const float4 w = *reinterpret_cast<const float4*>(wsm + (2 * i + h) * kF32Cols + q);
+      acc[i] = fmaf(x.x, w.x, fmaf(x.y, w.y, fmaf(x.z, w.z, fmaf(x.w, w.w, acc[i]))));
     }
     if (kGauss && (q >> 6) == h) {                        // half h of the features: sum x (ga x + gb)
       const float4 a = *reinterpret_cast<const float4*>(ga + q);
@@ -1251,7 +1250,7 @@ k_router_fwd_f32(const FwdParams p) {
   }
   float* pz = p.f32_part + static_cast<size_t>(tile * nck + ck) * (E + 1) * 128;
 #pragma unroll
-  for (int i = 0; i < kF32MaxE / 2; ++i) {
+  for (int i = 0; i < EB / 2; ++i) {
     const int e = 2 * i + h;
     if (e < E) pz[e * 128 + r] = acc[i];
   }
@@ -1366,9 +1365,17 @@ cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s) {
   const size_t smem = sizeof(float) * f32_smem_floats(p.dm) + sizeof(uint64_t) * kEpiBars + 64;
   if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
   const bool gauss = p.M_in == nullptr;
+  const int eb = round_up(p.dm.E, 16);
   return dispatch_km(p.dm.k, [&](auto km) -> cudaError_t {
     constexpr int KM = decltype(km)::value;
-    auto k = gauss ? k_router_fwd_f32<true, KM> : k_router_fwd_f32<false, KM>;
+    auto pick = [&](auto ebc) {
+      constexpr int EB = decltype(ebc)::value;
+      return gauss ? k_router_fwd_f32<true, KM, EB> : k_router_fwd_f32<false, KM, EB>;
+    };
+    auto k = eb <= 16 ? pick(std::integral_constant<int, 16>())
+           : eb <= 32 ? pick(std::integral_constant<int, 32>())
+           : eb <= 48 ? pick(std::integral_constant<int, 48>())
+                      : pick(std::integral_constant<int, 64>());
     cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(k, dim3(p.n_tiles * p.f32_chunks), dim3(256), smem, s, p);
