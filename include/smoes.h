@@ -198,6 +198,21 @@ smoes_status smoes_router_bwd(smoes_plan plan, const void* X, const void* W, con
                               float* dW, int accumulate_dW, void* dX, float* dlogits,
                               void* ws, size_t ws_bytes, cudaStream_t stream);
 
+/* (7) Bin-level load-balance loss (Sec. 3.5, eq. (16)) of the last forward on ws:
+ *     L_bal = sum_k N_B sum_{e in B_k} f_e P_e,
+ *   with U_k = the tokens that have at least one top-k expert in bin B_k, f_e = selections of e /
+ *   selections of all of B_k's experts, P_e = mean over U_k of g_je / sum_{e' in B_k} g_je' (the
+ *   gate renormalised inside the bin). A bin no token selects contributes 0. topk_idx [T, k]: the
+ *   forward's top-k. loss_bal [1] float32 receives L_bal (one layer); f_e, P_e [E] float32 or NULL.
+ *   The call also arms the backward: every smoes_router_bwd of this plan on the same ws until the
+ *   next forward adds the gradient of loss_scale * L_bal, taken with the counts f_e constant, to
+ *   the MI gradient (dlogits, dW and dX; topk_idx must then be passed to smoes_router_bwd). The
+ *   arming is tracked both on the host (the plan) and in ws (the forward kernels clear it).
+ *   Sums are fp32 per block of tokens and fp64 across blocks, in a fixed order. */
+smoes_status smoes_bin_balance(smoes_plan plan, const int32_t* topk_idx, float loss_scale,
+                               float* loss_bal, float* f_e, float* P_e, void* ws, size_t ws_bytes,
+                               cudaStream_t stream);
+
 /* (4) Bin-grouped permutation with de-duplicated dispatch (Sec. 4.5, "DeDup").
  *   One entry per unique (token, bin) pair, ordered by bin ascending then token ascending.
  *   topk_idx [T, k] int32 in [0, E). home [T] int32 in [0, n_bins) or NULL for the contiguous

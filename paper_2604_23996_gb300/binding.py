@@ -77,6 +77,7 @@ _sig = {
     "smoes_gaussian_stats_update": (_i, [_vp, _vp, _vp, C.c_double, _vp, _vp, _vp, _vp, _vp, _vp,
                                          _sz, _vp]),
     "smoes_adaptive_bins": (_i, [_vp, _vp, C.c_double, _vp, _vp, _vp, _vp]),
+    "smoes_bin_balance": (_i, [_vp, _vp, _f, _vp, _vp, _vp, _vp, _sz, _vp]),
 }
 for _name, (_res, _args) in _sig.items():
     _fn = getattr(_lib, _name)
@@ -215,6 +216,11 @@ def smoes_gaussian_stats_update(plan, X, is_vision, beta, N, S_mu, S_var, mu, va
     return _lib.smoes_gaussian_stats_update(plan, _p(X), _p(is_vision), float(beta), _p(N), _p(S_mu),
                                             _p(S_var), _p(mu), _p(var), _p(ws),
                                             ws.numel() * ws.element_size(), _stream(stream))
+
+
+def smoes_bin_balance(plan, topk_idx, loss_scale, loss_bal, ws, f_e=None, P_e=None, stream=None) -> int:
+    return _lib.smoes_bin_balance(plan, _p(topk_idx), float(loss_scale), _p(loss_bal), _p(f_e),
+                                  _p(P_e), _p(ws), ws.numel() * ws.element_size(), _stream(stream))
 
 
 def smoes_adaptive_bins(plan, expert_counts, beta, C_bar, expert_bin, f_spec=None, stream=None) -> int:

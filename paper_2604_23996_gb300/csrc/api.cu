@@ -24,7 +24,8 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 struct Layout {
   size_t status, sample_ticket, loss_ticket, offsets, token_sample, expert_bin, expert_slot,
       piece_base, sample_pieces, pieces, mi32, tabs, gsave, ginv, dw_part, dz_img, perm, attn_ticket, attn_part,
-      gcoef, perm_sync, fperm, stat_part, stat_nvis, stat_n0, f32_part, tile_ticket;
+      gcoef, perm_sync, fperm, stat_part, stat_nvis, stat_n0, f32_part, tile_ticket, bal_flag,
+      bal_f, bal_a, bal_h, bal_s, bal_u;
   size_t header_bytes;   // [0, header_bytes) is cleared by smoes_workspace_init
   size_t total;
 };
@@ -45,6 +46,7 @@ struct smoes_plan_s {
   int stat_blocks = 1;   // blocks of the statistics pass (one partial each)
   bool contig_bins = false;
   uint64_t limit_ns = kWaitLimitNs;   // bounded device waits
+  bool balance_armed = false;         // smoes_bin_balance enqueued since the last forward
   std::vector<int32_t> offsets, expert_bin, expert_slot, token_sample, piece_base, sample_pieces;
   Layout L{};
 };
@@ -78,6 +80,9 @@ WsView make_view(const smoes_plan_s* P, void* ws) {
   v.attn_part = reinterpret_cast<float*>(b + L.attn_part);
   v.gcoef = reinterpret_cast<float*>(b + L.gcoef);
   v.dcoef = P->dcoef;
+  v.bal_flag = reinterpret_cast<uint32_t*>(b + L.bal_flag);
+  v.bal_f = reinterpret_cast<float*>(b + L.bal_f);
+  v.bal_a = reinterpret_cast<float*>(b + L.bal_a);
   return v;
 }
 
@@ -182,6 +187,7 @@ smoes_status router_fwd(smoes_plan P, const void* X, const void* W, const float*
     return SMOES_ERR_ALIGNMENT;
   if (d.dtype == SMOES_F32 && d.E > 64) return SMOES_ERR_UNSUPPORTED;
 
+  P->balance_armed = false;           // the forward kernel clears the device flag too
   FwdParams p{};
   p.dm = make_dims(P);
   p.ws = make_view(P, ws);
@@ -338,6 +344,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.attn_ticket = take(sizeof(uint32_t) * (static_cast<size_t>(T) + 1));
   L.perm_sync = take(sizeof(uint32_t) * 4);
   L.tile_ticket = take(sizeof(uint32_t) * static_cast<size_t>(std::max(P->n_groups, 1)));
+  L.bal_flag = take(sizeof(uint32_t) * 4);
   L.header_bytes = o;
   L.offsets = take(sizeof(int32_t) * (B + 1));
   L.token_sample = take(sizeof(int32_t) * std::max(T, 1));
@@ -361,6 +368,11 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.stat_part = take(sizeof(float) * 4 * static_cast<size_t>(P->stat_blocks) * d.d);
   L.stat_nvis = take(sizeof(int32_t) * static_cast<size_t>(P->stat_blocks));
   L.stat_n0 = take(sizeof(double) * 2);
+  L.bal_f = take(sizeof(float) * E);
+  L.bal_a = take(sizeof(float) * K);
+  L.bal_h = take(sizeof(float) * static_cast<size_t>(P->stat_blocks) * E);
+  L.bal_s = take(sizeof(int32_t) * static_cast<size_t>(P->stat_blocks) * E);
+  L.bal_u = take(sizeof(int32_t) * static_cast<size_t>(P->stat_blocks) * K);
   L.f32_part = take(d.dtype == SMOES_F32 ? sizeof(float) * static_cast<size_t>(P->n_groups) *
                                                f32_chunks(d.d) * (E + 1) * 128 : 0);
   L.total = o;
@@ -567,6 +579,7 @@ smoes_status smoes_router_bwd(smoes_plan P, const void* X, const void* W, const 
   p.slice_width = P->bwd_slice_width;
   p.n_tiles = P->bwd_tiles;
   p.limit_ns = P->limit_ns;
+  p.balance_armed = P->balance_armed ? 1 : 0;
   cudaError_t e;
   if (d.dtype == SMOES_BF16) {
     const int E_pad = round_up(d.E, 64);
@@ -661,6 +674,44 @@ smoes_status smoes_gaussian_stats_update(smoes_plan P, const void* X, const uint
   p.nvis = reinterpret_cast<int32_t*>(b + P->L.stat_nvis);
   p.N0 = reinterpret_cast<double*>(b + P->L.stat_n0);
   return cuda_status(launch_stats_update(p, d.dtype == SMOES_BF16, stream));
+}
+
+smoes_status smoes_bin_balance(smoes_plan P, const int32_t* topk_idx, float loss_scale,
+                               float* loss_bal, float* f_e, float* P_e, void* ws, size_t ws_bytes,
+                               cudaStream_t stream) {
+  if (!P || !loss_bal) return SMOES_ERR_INVALID_ARG;
+  smoes_status st = check_ws(P, ws, ws_bytes);
+  if (st != SMOES_OK) return st;
+  const smoes_router_desc& d = P->desc;
+  if (d.T == 0) return cuda_status(cudaMemsetAsync(loss_bal, 0, sizeof(float), stream));
+  if (!topk_idx) return SMOES_ERR_INVALID_ARG;
+  if (!aligned16(topk_idx) || (f_e && !aligned16(f_e)) || (P_e && !aligned16(P_e)))
+    return SMOES_ERR_ALIGNMENT;
+  uint8_t* b = static_cast<uint8_t*>(ws);
+  WsView v = make_view(P, ws);
+  BalParams p{};
+  p.T = d.T;
+  p.E = d.E;
+  p.k = d.k;
+  p.K = d.n_bins;
+  p.N_B = P->N_B;
+  p.G = P->stat_blocks;
+  p.gsave = v.gsave;
+  p.topk_idx = topk_idx;
+  p.expert_bin = v.expert_bin;
+  p.scale = loss_scale;
+  p.part_h = reinterpret_cast<float*>(b + P->L.bal_h);
+  p.part_s = reinterpret_cast<int32_t*>(b + P->L.bal_s);
+  p.part_u = reinterpret_cast<int32_t*>(b + P->L.bal_u);
+  p.tab_f = v.bal_f;
+  p.tab_a = v.bal_a;
+  p.flag = v.bal_flag;
+  p.loss = loss_bal;
+  p.f_out = f_e;
+  p.P_out = P_e;
+  const smoes_status r = cuda_status(launch_bin_balance(p, stream));
+  if (r == SMOES_OK) P->balance_armed = true;
+  return r;
 }
 
 smoes_status smoes_adaptive_bins(smoes_plan P, const int32_t* expert_counts, double beta,

@@ -17,6 +17,8 @@
 // The per-group dW^T slice is written once at the end and summed over groups in fixed order.
 #include <cuda_bf16.h>
 
+#include <type_traits>
+
 #include "device_common.cuh"
 #include "ptx.cuh"
 #include "smoes_internal.cuh"
@@ -83,6 +85,46 @@ __device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
   return r;
 }
 
+// Gradient of the bin-level balance loss (eq. 16) at one token's logits, added to dz[N] of the
+// thread's N experts (g: their softmax scores, be: their bins (-1: none), fe: their f_e): for every
+// bin k the token routes to, dz_e += a_k h_e (f_e - sum_{e' in B_k} f_e' h_e') with h = g / (bin
+// sum). The bin sums run over the token's GS-lane thread group (xor shuffles); every lane takes
+// the same k iterations, and a bin repeated among the token's selections adds nothing again.
+template <int GS, int N>
+__device__ __forceinline__ void add_balance_grad(const BwdParams& p, int j, bool valid, const float (&g)[N],
+                                                 const int (&be)[N], const float (&fe)[N], float (&dz)[N]) {
+  const int k = p.dm.k;
+  int seen[kMaxTopK];
+#pragma unroll
+  for (int s = 0; s < kMaxTopK; ++s) {
+    if (s >= k) break;
+    const int es = valid ? __ldg(p.topk_idx + static_cast<size_t>(j) * k + s) : -1;
+    const int bs = (es >= 0 && es < p.dm.E) ? (p.dm.contig_bins ? es / p.dm.N_B : __ldg(p.ws.expert_bin + es)) : -1;
+    seen[s] = bs;
+    bool dup = bs < 0;
+#pragma unroll
+    for (int s2 = 0; s2 < kMaxTopK; ++s2)
+      if (s2 < s) dup = dup || seen[s2] == bs;
+    float v = 0.f, w = 0.f;
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+      v += be[i] == bs ? g[i] : 0.f;
+      w += be[i] == bs ? fe[i] * g[i] : 0.f;
+    }
+#pragma unroll
+    for (int o = 1; o < GS; o <<= 1) {
+      v += __shfl_xor_sync(0xffffffffu, v, o);
+      w += __shfl_xor_sync(0xffffffffu, w, o);
+    }
+    if (!dup && v > 0.f) {
+      const float a = __ldg(p.ws.bal_a + bs), iv = 1.f / v, phi = w * iv;
+#pragma unroll
+      for (int i = 0; i < N; ++i)
+        if (be[i] == bs) dz[i] = fmaf(a * g[i] * iv, fe[i] - phi, dz[i]);
+    }
+  }
+}
+
 // ------------------------------------------------------------------ dz preparation (bf16 path)
 // TPT = E_pad/8 threads per token, 8 experts each; the token's sum over experts is a shuffle
 // reduction inside its TPT-lane group. dz is written as the bf16 hi/lo pair (dz = hi + lo to
@@ -96,7 +138,7 @@ __device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
 // register budget otherwise).
 constexpr int kDzRep = 2;
 
-template <int TPT, bool kUp>
+template <int TPT, bool kUp, bool kBal>
 __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
   pdl_wait();                                         // scores and tables of the forward
   pdl_trigger();
@@ -120,6 +162,20 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
   float2 m[kDzRep];
   int smp[kDzRep];
   const bool vec = (E & 3) == 0 && e0 + 8 <= E;
+  // the balance term (eq. 16) when smoes_bin_balance armed this backward
+  const bool bal = kBal && p.topk_idx != nullptr && __ldcg(p.ws.bal_flag) != 0u;
+  int be[8];
+  float fe[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int e = e0 + i;
+    be[i] = -1;
+    fe[i] = 0.f;
+    if (bal && e < E) {
+      be[i] = dm.contig_bins ? e / dm.N_B : __ldg(p.ws.expert_bin + e);
+      fe[i] = __ldg(p.ws.bal_f + e);
+    }
+  }
 #pragma unroll
   for (int q = 0; q < kDzRep; ++q) {
     ga[q] = gb[q] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -185,6 +241,7 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
       for (int i = 0; i < 8; ++i)
         if (e0 + i < E) dz[i] += g[i] * (upstream_at(up, k, e0 + i) - up.gdt);
     }
+    if (kBal && bal) add_balance_grad<TPT, 8>(p, j[q], valid[q], g, be, fe, dz);
     if (valid[q] && p.dlogits) {
       float* dl = p.dlogits + static_cast<size_t>(j[q]) * E;
       if (vec) {
@@ -542,7 +599,10 @@ k_router_bwd_f32(const BwdParams p) {
     }
     part += __shfl_xor_sync(0xffffffffu, part, 1);
     part += __shfl_xor_sync(0xffffffffu, part, 2);
-    for (int e = qd; e < EB; e += 4) {
+    float dzv[EB / 4];
+#pragma unroll
+    for (int i = 0; i < EB / 4; ++i) {
+      const int e = qd + 4 * i;
       float v = 0.f;
       if (valid && e < E) {
         const int b = p.ws.expert_bin[e];
@@ -550,9 +610,27 @@ k_router_bwd_f32(const BwdParams p) {
         const float ge = g[e] * ginv;
         v = p.scale * ge * (u - part);
         if (has_up) v += ge * (upstream_at(up, k, e) - up.gdt);
-        if (p.dlogits && ck == 0) p.dlogits[static_cast<size_t>(j) * E + e] = v;
       }
-      dzs[r * kZs + e] = v;
+      dzv[i] = v;
+    }
+    if (p.topk_idx && __ldcg(p.ws.bal_flag) != 0u) {   // the balance term (eq. 16); block-uniform
+      float gq[EB / 4], fq[EB / 4];
+      int bq[EB / 4];
+#pragma unroll
+      for (int i = 0; i < EB / 4; ++i) {
+        const int e = qd + 4 * i;
+        const bool in = valid && e < E;
+        gq[i] = in ? g[e] * ginv : 0.f;
+        bq[i] = in ? p.ws.expert_bin[e] : -1;
+        fq[i] = in ? p.ws.bal_f[e] : 0.f;
+      }
+      add_balance_grad<4, EB / 4>(p, j, valid, gq, bq, fq, dzv);
+    }
+#pragma unroll
+    for (int i = 0; i < EB / 4; ++i) {
+      const int e = qd + 4 * i;
+      if (valid && e < E && p.dlogits && ck == 0) p.dlogits[static_cast<size_t>(j) * E + e] = dzv[i];
+      dzs[r * kZs + e] = dzv[i];
     }
   }
   const float* X = static_cast<const float*>(p.X);
@@ -678,13 +756,16 @@ cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s) {
   const int tokens_per_block = kDzRep * 256 / (E_pad / 8);
   const long rows = static_cast<long>(p.n_tiles) * kBwdBT;
   const int blocks = static_cast<int>((rows + tokens_per_block - 1) / tokens_per_block);
-  const bool up = p.d_topk_w != nullptr;
-  if (E_pad == 64)
-    return up ? launch_pdl(k_dz_prep<8, true>, dim3(blocks), dim3(256), 0, s, p)
-              : launch_pdl(k_dz_prep<8, false>, dim3(blocks), dim3(256), 0, s, p);
-  if (E_pad == 128)
-    return up ? launch_pdl(k_dz_prep<16, true>, dim3(blocks), dim3(256), 0, s, p)
-              : launch_pdl(k_dz_prep<16, false>, dim3(blocks), dim3(256), 0, s, p);
+  // the upstream-gradient and balance variants keep their tables out of the common kernel's
+  // registers; the balance variant still checks the arming flag on the device
+  const bool up = p.d_topk_w != nullptr, bal = p.balance_armed != 0;
+  auto pick = [&](auto tpt) {
+    constexpr int TPT = decltype(tpt)::value;
+    return up ? (bal ? k_dz_prep<TPT, true, true> : k_dz_prep<TPT, true, false>)
+              : (bal ? k_dz_prep<TPT, false, true> : k_dz_prep<TPT, false, false>);
+  };
+  if (E_pad == 64) return launch_pdl(pick(std::integral_constant<int, 8>()), dim3(blocks), dim3(256), 0, s, p);
+  if (E_pad == 128) return launch_pdl(pick(std::integral_constant<int, 16>()), dim3(blocks), dim3(256), 0, s, p);
   return cudaErrorInvalidValue;
 }
 

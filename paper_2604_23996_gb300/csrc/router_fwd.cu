@@ -887,6 +887,7 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
   // X, W, the statistics and the outputs may be in use by the kernel before this one
   pdl_wait();
   pdl_trigger();
+  if (blockIdx.x == 0 && threadIdx.x == 0) *p.ws.bal_flag = 0u;   // a new forward: no balance term yet
 
   if (kGauss && warp >= 2 && warp < 10) {
     // this CTA's Gaussian coefficients (eqs. 8-9), float4 {ga[2i], ga[2i+1], gb[2i], gb[2i+1]}
@@ -1193,6 +1194,7 @@ k_router_fwd_f32(const FwdParams p) {
   const int t = threadIdx.x, r = t & 127, h = t >> 7;
   pdl_wait();
   pdl_trigger();
+  if (blockIdx.x == 0 && t == 0) *p.ws.bal_flag = 0u;             // a new forward: no balance term yet
   const float* X = static_cast<const float*>(p.X);
   const float* W = static_cast<const float*>(p.W);
   // the tile's 128 x 128 block of X and the [E, 128] block of W, zero past T and d

@@ -52,6 +52,11 @@ struct WsView {
   float* attn_part;          // [H_max * T] per-head vision mass
   float* gcoef;              // Gaussian score coefficients: ga[dcoef], gb[dcoef], part[dcoef/256]
   int dcoef;                 // round_up(d, 256)
+  // bin-level load balance (eq. 16): the backward adds its gradient while *bal_flag != 0 (set by
+  // smoes_bin_balance, cleared by every forward); bal_f [E] = f_e, bal_a [K] = scale N_B / |U_k|
+  uint32_t* bal_flag;
+  float* bal_f;
+  float* bal_a;
 };
 
 struct Dims {
@@ -119,6 +124,7 @@ struct BwdParams {
   int slice_width;           // columns per d-slice
   int n_tiles;               // token tiles
   uint64_t limit_ns;
+  int balance_armed;         // host's view: smoes_bin_balance was called since the last forward
 };
 
 struct PermParams {
@@ -186,6 +192,26 @@ struct StatsParams {
   float* part;
   int32_t* nvis;
   double* N0;                // [2] copy of N_{t-1}
+};
+
+// Bin-level load-balance loss (eq. 16) from the forward's saved scores: per-block partials
+// part_h [G][E] (sums of the bin-renormalised gate over the bin's routed tokens), part_s [G][E]
+// (selections), part_u [G][K] (routed tokens per bin), then f, P, the loss and the table.
+struct BalParams {
+  int T, E, k, K, N_B, G;
+  const float* gsave;
+  const int32_t* topk_idx;
+  const int32_t* expert_bin;
+  double scale;
+  float* part_h;
+  int32_t* part_s;
+  int32_t* part_u;
+  float* tab_f;
+  float* tab_a;
+  uint32_t* flag;
+  float* loss;
+  float* f_out;              // [E] or null
+  float* P_out;              // [E] or null
 };
 
 // Momentum-adaptive binning (eqs. 10-11).
@@ -260,6 +286,7 @@ cudaError_t launch_gauss_coef(const float* mu, const float* var, int d, int dcoe
                               uint32_t* status, cudaStream_t s);
 cudaError_t launch_stats_update(const StatsParams& p, bool bf16, cudaStream_t s);
 cudaError_t launch_adaptive_bins(const BinsParams& p, cudaStream_t s);
+cudaError_t launch_bin_balance(const BalParams& p, cudaStream_t s);
 cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                              int n_sms, cudaStream_t s);
 
