@@ -64,6 +64,43 @@ def gaussian_score(X, mu, var, tau):
     return e / e.sum(axis=1, keepdims=True)
 
 
+def gmm_log_likelihood(X, log_pi, mu, var):
+    """Log-likelihood of every token under each modality's diagonal Gaussian mixture: the
+    estimator the paper explores beyond the single Gaussian of eq. (8) (supplementary, "GMM
+    estimator" with k components).
+
+    LL[j, m] = log sum_c pi[m, c] N(x_j; mu[m, c], diag var[m, c])
+             = logsumexp_c ( log pi[m, c] - 1/2 sum_d ( log(2 pi) + log var[m, c, d]
+                                                       + (x_jd - mu[m, c, d])^2 / var[m, c, d] ) ).
+    The log(2 pi) term is the same for both modalities and is kept so that the values are true
+    log-densities (it cancels in the score).
+
+    X [T, d]; log_pi [2, C]; mu, var [2, C, d] -> LL [T, 2].
+    """
+    X, log_pi, mu, var = _f64(X), _f64(log_pi), _f64(mu), _f64(var)
+    T, d = X.shape
+    C = mu.shape[1]
+    LL = np.empty((T, 2))
+    for m in range(2):
+        q = np.empty((T, C))
+        for c in range(C):
+            q[:, c] = log_pi[m, c] - 0.5 * np.sum(np.log(2.0 * np.pi) + np.log(var[m, c])[None, :]
+                                                  + (X - mu[m, c][None, :]) ** 2 / var[m, c][None, :],
+                                                  axis=1)
+        top = q.max(axis=1, keepdims=True)
+        LL[:, m] = top[:, 0] + np.log(np.sum(np.exp(q - top), axis=1))
+    return LL
+
+
+def gmm_score(X, log_pi, mu, var, tau):
+    """Soft modality score with the GMM estimator: eq. (9) applied to the mixture
+    log-likelihoods of gmm_log_likelihood (C = 1 gives the Gaussian score of eqs. 8-9)."""
+    LL = gmm_log_likelihood(X, log_pi, mu, var) / float(tau)
+    LL = LL - LL.max(axis=1, keepdims=True)
+    e = np.exp(LL)
+    return e / e.sum(axis=1, keepdims=True)
+
+
 def attention_vision_mass(Q, K, m_keys, sm_scale, causal=True, key_bias=None, queries=None):
     """Attention-accumulated vision score, eqs. (2)-(3).
 
@@ -182,6 +219,48 @@ def topk_route(z, g, k, renorm=False):
     if renorm:
         w = w / w.sum(axis=1, keepdims=True)
     return order.astype(np.int32), w
+
+
+def sigmoid_gate(z, score_bias=None, k=None):
+    """Sigmoid router with a selection bias (the router of Moonlight-MoE in the paper's backbone
+    table): affinities s = sigmoid(z); experts chosen by the top-k of s + b (the bias only steers
+    the choice); top-k weights s / sum of the chosen s. Readings: the gating scores g that enter
+    eq. (12) (and the bin sums) are the affinities normalised over all experts, g = s / sum_e s,
+    so that p_j. is a distribution as with the softmax router; ties in s + b go to the lower
+    expert index.
+
+    z [T, E]; score_bias [E] or None. Returns dict(s, g, topk_idx [T, k] int32, topk_w [T, k]).
+    """
+    z = _f64(z)
+    s = 1.0 / (1.0 + np.exp(-z))
+    g = s / s.sum(axis=1, keepdims=True)
+    out = dict(s=s, g=g)
+    if k is not None:
+        key = s + (0.0 if score_bias is None else _f64(score_bias)[None, :])
+        idx = np.argsort(-key, axis=1, kind='stable')[:, :k]
+        w = np.take_along_axis(s, idx, axis=1)
+        out.update(topk_idx=idx.astype(np.int32), topk_w=w / w.sum(axis=1, keepdims=True))
+    return out
+
+
+def sigmoid_grad_logits(s, dL_dg):
+    """Gradient at the logits of a loss given through g = s / sum s, s = sigmoid(z):
+    dL/dz_e = s_e (1 - s_e) (dL/dg_e - sum_e' g_e' dL/dg_e') / sum s."""
+    s, dL_dg = _f64(s), _f64(dL_dg)
+    S = s.sum(axis=1, keepdims=True)
+    g = s / S
+    return s * (1.0 - s) * (dL_dg - np.sum(g * dL_dg, axis=1, keepdims=True)) / S
+
+
+def topk_masked_gate(g, topk_idx):
+    """The top-k-masked reading of g in eq. (12): the gate restricted to the chosen experts and
+    renormalised over them (zero elsewhere), so that its bin sums still form a distribution."""
+    g = _f64(g)
+    out = np.zeros_like(g)
+    idx = np.asarray(topk_idx, dtype=np.int64)
+    sel = np.take_along_axis(g, idx, axis=1)
+    np.put_along_axis(out, idx, sel / sel.sum(axis=1, keepdims=True), axis=1)
+    return out
 
 
 def bin_probs(g, expert_bin, n_bins):
