@@ -50,7 +50,8 @@ typedef enum { SMOES_F32 = 0, SMOES_BF16 = 1 } smoes_dtype;
 typedef enum {
   SMOES_SCORE_PROVIDED = 0,       /* M is given by the caller                       */
   SMOES_SCORE_GAUSS = 1,          /* Gaussian-statistics score, eqs. (8)-(9)        */
-  SMOES_SCORE_ATTN = 2            /* attention-accumulated score, eqs. (2)-(4)      */
+  SMOES_SCORE_ATTN = 2,           /* attention-accumulated score, eqs. (2)-(4)      */
+  SMOES_SCORE_GMM = 3             /* Gaussian-mixture estimator (supplementary)     */
 } smoes_score_mode;
 
 typedef struct smoes_plan_s* smoes_plan;
@@ -109,9 +110,25 @@ typedef struct {
   const float* x_norm;
 } smoes_attn_args;
 
+/* Gaussian-mixture score inputs (the estimator the paper explores beyond eq. (8)): each
+ *   modality's features follow n_components (1..4) diagonal Gaussians with weights pi.
+ *   X [T, d] (plan dtype); log_pi [2, C] float32 (log weights, each row summing to 1 in the
+ *   linear domain); mu, var [2, C, d] float32, var > 0; tau as for smoes_gauss_args.
+ *   M_v = sigmoid((LL_v - LL_t) / tau) with LL_m = log sum_c pi_mc N(x; mu_mc, var_mc);
+ *   n_components = 1 gives the score of eqs. (8)-(9). */
+typedef struct {
+  const void* X;
+  int n_components;
+  const float* log_pi;
+  const float* mu;
+  const float* var;
+  float tau;
+} smoes_gmm_args;
+
 typedef struct {
   smoes_gauss_args gauss;
   smoes_attn_args attn;
+  smoes_gmm_args gmm;
 } smoes_score_args;
 
 /* Validates the descriptor and builds the host-side plan (no device memory is touched).
@@ -147,6 +164,8 @@ smoes_status smoes_read_device_status(smoes_plan plan, const void* ws, cudaStrea
  *   mode SMOES_SCORE_GAUSS: M[j] = softmax_m(LL[j, m] / tau) with LL of eq. (8).
  *   mode SMOES_SCORE_ATTN:  M[j, 0] = (1/H) sum_h sum_j' softmax_j'(s q.k_j' + bias_j') m_j'
  *                           (eq. (3), optionally followed by eq. (4)); M[j, 1] = 1 - M[j, 0].
+ *   mode SMOES_SCORE_GMM:   eq. (9) on the Gaussian-mixture log-likelihoods of args->gmm
+ *                           (n_components > 4 returns SMOES_ERR_UNSUPPORTED).
  *   M: [T, 2] float32 output. ws is needed by SMOES_SCORE_ATTN (head partial sums). */
 smoes_status smoes_modality_score(smoes_plan plan, smoes_score_mode mode,
                                   const smoes_score_args* args, float* M,

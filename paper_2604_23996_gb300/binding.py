@@ -24,7 +24,7 @@ STATUS_NAMES = {0: "SMOES_OK", -1: "SMOES_ERR_INVALID_ARG", -2: "SMOES_ERR_UNSUP
                 -3: "SMOES_ERR_ALIGNMENT", -4: "SMOES_ERR_WORKSPACE", -5: "SMOES_ERR_CUDA",
                 -6: "SMOES_ERR_DEVICE_TIMEOUT", -7: "SMOES_ERR_DATA"}
 SMOES_F32, SMOES_BF16 = 0, 1
-SMOES_SCORE_PROVIDED, SMOES_SCORE_GAUSS, SMOES_SCORE_ATTN = 0, 1, 2
+SMOES_SCORE_PROVIDED, SMOES_SCORE_GAUSS, SMOES_SCORE_ATTN, SMOES_SCORE_GMM = 0, 1, 2, 3
 
 
 class SmoesError(RuntimeError):
@@ -52,8 +52,13 @@ class AttnArgs(C.Structure):
                 ("xattn_norm", C.c_void_p), ("x_norm", C.c_void_p)]
 
 
+class GmmArgs(C.Structure):
+    _fields_ = [("X", C.c_void_p), ("n_components", C.c_int), ("log_pi", C.c_void_p),
+                ("mu", C.c_void_p), ("var", C.c_void_p), ("tau", C.c_float)]
+
+
 class ScoreArgs(C.Structure):
-    _fields_ = [("gauss", GaussArgs), ("attn", AttnArgs)]
+    _fields_ = [("gauss", GaussArgs), ("attn", AttnArgs), ("gmm", GmmArgs)]
 
 
 _vp, _i, _f, _sz = C.c_void_p, C.c_int, C.c_float, C.c_size_t
@@ -144,7 +149,7 @@ def smoes_read_device_status(plan, ws: torch.Tensor, stream=None):
 
 
 def smoes_modality_score(plan, mode, M, ws, X=None, mu=None, var=None, tau=0.0, attn=None,
-                         stream=None) -> int:
+                         gmm=None, stream=None) -> int:
     """attn: dict with Q, K, B, H, S, hd, is_vision | m_prev, key_bias, sm_scale, causal,
     xattn_norm, x_norm (tensors or scalars)."""
     args = ScoreArgs()
@@ -155,6 +160,9 @@ def smoes_modality_score(plan, mode, M, ws, X=None, mu=None, var=None, tau=0.0, 
                              _p(a.get("is_vision")), _p(a.get("m_prev")), _p(a.get("key_bias")),
                              float(a["sm_scale"]), int(a.get("causal", 1)),
                              _p(a.get("xattn_norm")), _p(a.get("x_norm")))
+    if gmm is not None:
+        args.gmm = GmmArgs(_p(gmm["X"]), int(gmm["n_components"]), _p(gmm["log_pi"]), _p(gmm["mu"]),
+                           _p(gmm["var"]), float(gmm.get("tau", 0.0)))
     return _lib.smoes_modality_score(plan, mode, C.byref(args), _p(M), _p(ws),
                                      ws.numel() * ws.element_size(), _stream(stream))
 

@@ -25,7 +25,7 @@ struct Layout {
   size_t status, sample_ticket, loss_ticket, offsets, token_sample, expert_bin, expert_slot,
       piece_base, sample_pieces, pieces, mi32, tabs, gsave, ginv, dw_part, dz_img, perm, attn_ticket, attn_part,
       gcoef, perm_sync, fperm, stat_part, stat_nvis, stat_n0, f32_part, tile_ticket, bal_flag,
-      bal_f, bal_a, bal_h, bal_s, bal_u;
+      bal_f, bal_a, bal_h, bal_s, bal_u, gmmcoef;
   size_t header_bytes;   // [0, header_bytes) is cleared by smoes_workspace_init
   size_t total;
 };
@@ -368,6 +368,7 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   L.stat_part = take(sizeof(float) * 4 * static_cast<size_t>(P->stat_blocks) * d.d);
   L.stat_nvis = take(sizeof(int32_t) * static_cast<size_t>(P->stat_blocks));
   L.stat_n0 = take(sizeof(double) * 2);
+  L.gmmcoef = take(sizeof(float) * kGmmMaxForms * (2 * static_cast<size_t>(P->dcoef) + P->dcoef / 256));
   L.bal_f = take(sizeof(float) * E);
   L.bal_a = take(sizeof(float) * K);
   L.bal_h = take(sizeof(float) * static_cast<size_t>(P->stat_blocks) * E);
@@ -451,6 +452,32 @@ smoes_status smoes_modality_score(smoes_plan P, smoes_score_mode mode, const smo
     cudaError_t e = launch_gauss_coef(g.mu, g.var, d.d, v.dcoef, v.gcoef, v.status, stream);
     if (e == cudaSuccess) e = launch_gauss_score(p, d.dtype, P->n_sms, stream);
     return cuda_status(e);
+  }
+  if (mode == SMOES_SCORE_GMM) {
+    const smoes_gmm_args& g = args->gmm;
+    if (!g.X || !g.log_pi || !g.mu || !g.var) return SMOES_ERR_INVALID_ARG;
+    if (g.n_components < 1) return SMOES_ERR_INVALID_ARG;
+    if (g.n_components > kGmmMaxComponents) return SMOES_ERR_UNSUPPORTED;
+    // the forms' coefficients stay in shared memory: 2 (2C - 1) round_up(d, 256) floats
+    if (sizeof(float) * 2 * (2 * g.n_components - 1) * static_cast<size_t>(round_up(d.d, 256)) > 227u * 1024u)
+      return SMOES_ERR_UNSUPPORTED;
+    if (!aligned16(g.X)) return SMOES_ERR_ALIGNMENT;
+    if (d.T == 0) return SMOES_OK;
+    GmmParams p{};
+    p.T = d.T;
+    p.d = d.d;
+    p.C = g.n_components;
+    p.F = 2 * g.n_components - 1;
+    p.dcoef = v.dcoef;
+    p.X = g.X;
+    p.log_pi = g.log_pi;
+    p.mu = g.mu;
+    p.var = g.var;
+    p.inv_tau = 1.f / (g.tau > 0.f ? g.tau : 0.5f * d.d);
+    p.coef = reinterpret_cast<float*>(static_cast<uint8_t*>(ws) + P->L.gmmcoef);
+    p.M = M;
+    p.status = v.status;
+    return cuda_status(launch_gmm_score(p, d.dtype, P->n_sms, stream));
   }
   if (mode == SMOES_SCORE_ATTN) {
     const smoes_attn_args& a = args->attn;

@@ -157,6 +157,21 @@ struct GaussParams {
   uint32_t* status;
 };
 
+// Gaussian-mixture score: C components per modality, F = 2C - 1 forms relative to (text, 0).
+constexpr int kGmmMaxComponents = 4;
+constexpr int kGmmMaxForms = 2 * kGmmMaxComponents - 1;
+struct GmmParams {
+  int T, d, C, F, dcoef;
+  const void* X;
+  const float* log_pi;       // [2, C]
+  const float* mu;           // [2, C, d]
+  const float* var;          // [2, C, d]
+  float inv_tau;
+  float* coef;               // workspace: [F][2][dcoef] + [F][dcoef / 256]
+  float* M;
+  uint32_t* status;
+};
+
 struct AttnParams {
   int B, H, S, hd, T;
   const void* Q;
@@ -287,6 +302,7 @@ cudaError_t launch_gauss_coef(const float* mu, const float* var, int d, int dcoe
 cudaError_t launch_stats_update(const StatsParams& p, bool bf16, cudaStream_t s);
 cudaError_t launch_adaptive_bins(const BinsParams& p, cudaStream_t s);
 cudaError_t launch_bin_balance(const BalParams& p, cudaStream_t s);
+cudaError_t launch_gmm_score(const GmmParams& p, smoes_dtype dt, int n_sms, cudaStream_t s);
 cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                              int n_sms, cudaStream_t s);
 
