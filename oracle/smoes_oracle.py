@@ -492,6 +492,84 @@ def router_backward(X, W, M, fwd, expert_bin, sample_offsets, loss_scale, d_topk
     return dz, dW, dX
 
 
+def mi_grad_gate(M, expert_bin, sample_offsets, tabs, loss_scale, N_B):
+    """Gradient of loss_scale * L_MI with respect to the gate values that enter eq. (12) (the
+    quantity summed into the bins): -(loss_scale / B) u[j, bin(e)], with u as in mi_grad_logits.
+    Returns [T, E]."""
+    M = _f64(M)
+    expert_bin = np.asarray(expert_bin)
+    offs = np.asarray(sample_offsets)
+    B = len(offs) - 1
+    out = np.zeros((M.shape[0], len(expert_bin)))
+    for i in range(B):
+        s, e = int(offs[i]), int(offs[i + 1])
+        tab = tabs[i]
+        K = tab['P'].shape[1]
+        u_coef = np.zeros((2, K))
+        for m in range(2):
+            if tab['A'][m] > MASS_EPS:
+                with np.errstate(divide='ignore', invalid='ignore'):
+                    ratio = np.where(tab['P'][m] > 0, tab['P'][m] / (tab['Pm'][m] * tab['Pk']), 1.0)
+                u_coef[m] = (np.log(ratio) - tab['I']) / tab['Z'] / (N_B * tab['A'][m])
+        out[s:e] = -(loss_scale / B) * (M[s:e] @ u_coef)[:, expert_bin]
+    return out
+
+
+def softmax_grad_logits(g, dL_dg):
+    """Chain rule through g = softmax(z): dL/dz = g (dL/dg - sum_e' g_e' dL/dg_e')."""
+    g, dL_dg = _f64(g), _f64(dL_dg)
+    return g * (dL_dg - np.sum(g * dL_dg, axis=1, keepdims=True))
+
+
+def masked_gate_grad(g, topk_idx, dL_dgt):
+    """Chain rule through the top-k-masked gate gt = g / sum_sel g on the chosen experts:
+    dL/dg_e = (dL/dgt_e - sum_sel gt dL/dgt) / sum_sel g for chosen e, 0 elsewhere."""
+    g, dL_dgt = _f64(g), _f64(dL_dgt)
+    idx = np.asarray(topk_idx, dtype=np.int64)
+    gs = np.take_along_axis(g, idx, axis=1)
+    G = gs.sum(axis=1, keepdims=True)
+    ds = np.take_along_axis(dL_dgt, idx, axis=1)
+    out = np.zeros_like(g)
+    np.put_along_axis(out, idx, (ds - np.sum(gs / G * ds, axis=1, keepdims=True)) / G, axis=1)
+    return out
+
+
+def router_forward_variant(X, W, M, expert_bin, n_bins, sample_offsets, k, gate='softmax',
+                           score_bias=None, mask=False, renorm=False):
+    """Forward of one router layer for the router variants of the backbone table and of the
+    readings of eq. (12): gate 'softmax' (Sec. 3.1) or 'sigmoid' (sigmoid_gate, with an optional
+    selection bias; its top-k weights are always renormalised), and the gate entering eq. (12)
+    either dense (all experts) or top-k-masked (topk_masked_gate). Same outputs as
+    router_forward plus 'gq', the gate values summed into the bins, and 's' (sigmoid only)."""
+    z = gate_logits(X, W)
+    if gate == 'softmax':
+        g = softmax_gate(z)
+        idx, w = topk_route(z, g, k, renorm)
+        s = None
+    elif gate == 'sigmoid':
+        out = sigmoid_gate(z, score_bias, k)
+        g, idx, w, s = out['g'], out['topk_idx'], out['topk_w'], out['s']
+    else:
+        raise ValueError(gate)
+    gq = topk_masked_gate(g, idx) if mask else g
+    N_B = len(expert_bin) // n_bins
+    p = bin_probs(gq, expert_bin, n_bins)
+    mis, joint, loss, tabs = mi_loss(_f64(M), p, sample_offsets, N_B)
+    return dict(z=z, g=g, s=s, gq=gq, topk_idx=idx, topk_w=w, p=p, mi=mis, joint=joint, loss=loss,
+                tabs=tabs, gate=gate, mask=mask)
+
+
+def router_backward_variant(X, W, M, fwd, expert_bin, sample_offsets, loss_scale):
+    """Backward of loss_scale * L_MI for router_forward_variant: dL/d(gate values of eq. 12)
+    (mi_grad_gate), through the top-k mask when used (masked_gate_grad), then through the gate
+    (softmax_grad_logits or sigmoid_grad_logits); dW = dz^T X, dX = dz W."""
+    N_B = len(expert_bin) // fwd['p'].shape[1]
+    dgq = mi_grad_gate(M, expert_bin, sample_offsets, fwd['tabs'], loss_scale, N_B)
+    dg = masked_gate_grad(fwd['g'], fwd['topk_idx'], dgq) if fwd['mask'] else dgq
+    dz = softmax_grad_logits(fwd['g'], dg) if fwd['gate'] == 'softmax' else sigmoid_grad_logits(fwd['s'], dg)
+    return dz, dz.T @ _f64(X), dz @ _f64(W)
+
+
 def msi(expert_counts):
     """Modality Specialization Index, eqs. (18)-(19), for one layer from counts C [2, E]
     (row 0 vision, row 1 text). Returns a value in [0, 1]."""

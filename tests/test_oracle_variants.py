@@ -104,3 +104,59 @@ def test_topk_masked_gate_is_the_renormalised_topk_weight():
     mask = np.zeros_like(g, dtype=bool)
     np.put_along_axis(mask, idx.astype(np.int64), True, axis=1)
     assert np.all(gm[~mask] == 0.0)
+
+
+def _variant_case(seed, T=16, d=6, E=8, n_bins=4, offs=(0, 7, 16)):
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((T, d))
+    W = 0.5 * rng.standard_normal((E, d))
+    Mv = rng.uniform(0.05, 0.95, T)
+    M = np.stack([Mv, 1 - Mv], axis=1)
+    eb = np.arange(E) // (E // n_bins)
+    return X, W, M, eb, n_bins, np.array(offs)
+
+
+def test_default_variant_is_the_pinned_router():
+    X, W, M, eb, K, offs = _variant_case(10)
+    a = O.router_forward(X, W, M, eb, K, offs, 3)
+    b = O.router_forward_variant(X, W, M, eb, K, offs, 3)
+    np.testing.assert_array_equal(a["topk_idx"], b["topk_idx"])
+    np.testing.assert_allclose(b["mi"], a["mi"], rtol=1e-14, atol=1e-16)
+    dz_a, dW_a, _ = O.router_backward(X, W, M, a, eb, offs, 0.8)
+    dz_b, dW_b, _ = O.router_backward_variant(X, W, M, b, eb, offs, 0.8)
+    np.testing.assert_allclose(dz_b, dz_a, rtol=1e-12, atol=1e-16)
+    np.testing.assert_allclose(dW_b, dW_a, rtol=1e-12, atol=1e-16)
+
+
+@pytest.mark.parametrize("gate,mask", [("softmax", True), ("sigmoid", False), ("sigmoid", True)])
+def test_variant_gradient_central_differences(gate, mask):
+    X, W, M, eb, K, offs = _variant_case(11)
+    bias = np.linspace(-0.3, 0.3, W.shape[0]) if gate == "sigmoid" else None
+    k = 3
+    f0 = O.router_forward_variant(X, W, M, eb, K, offs, k, gate=gate, score_bias=bias, mask=mask)
+    _, dW, dX = O.router_backward_variant(X, W, M, f0, eb, offs, 1.0)
+
+    def loss(Xv, Wv):
+        f = O.router_forward_variant(Xv, Wv, M, eb, K, offs, k, gate=gate, score_bias=bias, mask=mask)
+        assert np.array_equal(f["topk_idx"], f0["topk_idx"])     # the choice is locally constant
+        return f["loss"]
+
+    h = 1e-6
+    for A, grad, name in ((W, dW, "W"), (X, dX, "X")):
+        num = np.zeros_like(A)
+        for idx in np.ndindex(*A.shape):
+            Ap, Am = A.copy(), A.copy()
+            Ap[idx] += h
+            Am[idx] -= h
+            num[idx] = ((loss(Xv=X, Wv=Ap) - loss(Xv=X, Wv=Am)) if name == "W"
+                        else (loss(Xv=Ap, Wv=W) - loss(Xv=Am, Wv=W))) / (2 * h)
+        np.testing.assert_allclose(grad, num, rtol=2e-5, atol=5e-10, err_msg=f"{gate} mask={mask} d{name}")
+
+
+def test_masked_bins_hold_only_chosen_experts():
+    X, W, M, eb, K, offs = _variant_case(12)
+    f = O.router_forward_variant(X, W, M, eb, K, offs, 2, mask=True)
+    np.testing.assert_allclose(f["p"].sum(axis=1), 1.0, rtol=1e-14)
+    chosen_bins = eb[f["topk_idx"]]
+    for j in range(X.shape[0]):
+        assert set(np.nonzero(f["p"][j] > 0)[0]) == set(chosen_bins[j])
