@@ -535,12 +535,14 @@ def masked_gate_grad(g, topk_idx, dL_dgt):
 
 
 def router_forward_variant(X, W, M, expert_bin, n_bins, sample_offsets, k, gate='softmax',
-                           score_bias=None, mask=False, renorm=False):
+                           score_bias=None, mask=False, renorm=False, topk_idx=None):
     """Forward of one router layer for the router variants of the backbone table and of the
     readings of eq. (12): gate 'softmax' (Sec. 3.1) or 'sigmoid' (sigmoid_gate, with an optional
     selection bias; its top-k weights are always renormalised), and the gate entering eq. (12)
     either dense (all experts) or top-k-masked (topk_masked_gate). Same outputs as
-    router_forward plus 'gq', the gate values summed into the bins, and 's' (sigmoid only)."""
+    router_forward plus 'gq', the gate values summed into the bins, and 's' (sigmoid only).
+    topk_idx: a given choice instead of the gate's own (stage-wise comparisons of what follows
+    the choice); the weights are then those of the given experts."""
     z = gate_logits(X, W)
     if gate == 'softmax':
         g = softmax_gate(z)
@@ -551,6 +553,12 @@ def router_forward_variant(X, W, M, expert_bin, n_bins, sample_offsets, k, gate=
         g, idx, w, s = out['g'], out['topk_idx'], out['topk_w'], out['s']
     else:
         raise ValueError(gate)
+    if topk_idx is not None:
+        idx = np.asarray(topk_idx).astype(np.int32)
+        src = g if gate == 'softmax' else s
+        w = np.take_along_axis(src, idx.astype(np.int64), axis=1)
+        if gate == 'sigmoid' or renorm:
+            w = w / w.sum(axis=1, keepdims=True)
     gq = topk_masked_gate(g, idx) if mask else g
     N_B = len(expert_bin) // n_bins
     p = bin_probs(gq, expert_bin, n_bins)
@@ -696,6 +704,48 @@ def bin_balance_loss(g, topk_idx, expert_bin, n_bins):
         P[members] = np.mean(gk / gk.sum(axis=1, keepdims=True), axis=0)
         L += N_B * float(np.sum(f[members] * P[members]))
     return L, dict(f=f, P=P, used=used)
+
+
+def sigmoid_topk_weight_grad_logits(s, topk_idx, d_topk_w):
+    """Gradient reaching the logits from an upstream gradient of the sigmoid router's top-k
+    weights w_i = s_i / sum_chosen s: for a chosen expert e, dL/ds_e = (d_e - sum_i w_i d_i) /
+    sum_chosen s, then dL/dz_e = s_e (1 - s_e) dL/ds_e; zero for the others."""
+    s = _f64(s)
+    idx = np.asarray(topk_idx, dtype=np.int64)
+    d = _f64(d_topk_w)
+    ss = np.take_along_axis(s, idx, axis=1)
+    S = ss.sum(axis=1, keepdims=True)
+    w = ss / S
+    ds = (d - np.sum(w * d, axis=1, keepdims=True)) / S
+    out = np.zeros_like(s)
+    np.put_along_axis(out, idx, ss * (1.0 - ss) * ds, axis=1)
+    return out
+
+
+def bin_balance_grad_gate(g, topk_idx, expert_bin, n_bins, scale):
+    """Gradient of scale * L_bal (eq. 16) with respect to the gate values g (f_e constant), the
+    quantity bin_balance_grad_logits pushes through the softmax:
+        dL/dg_je = N_B / |U_k| * (f_e - sum_{e' in B_k} f_e' h_je') / G_jk  (j in U_k, e in B_k)."""
+    g = _f64(g)
+    T, E = g.shape
+    eb = np.asarray(expert_bin)
+    N_B = E // n_bins
+    _, parts = bin_balance_loss(g, topk_idx, expert_bin, n_bins)
+    f = parts["f"]
+    sel = np.zeros((T, E), dtype=bool)
+    sel[np.arange(T)[:, None], np.asarray(topk_idx)] = True
+    dg = np.zeros((T, E))
+    for k in range(n_bins):
+        if not parts["used"][k]:
+            continue
+        members = np.nonzero(eb == k)[0]
+        U = sel[:, members].any(axis=1)
+        gk = g[U][:, members]
+        G = gk.sum(axis=1, keepdims=True)
+        h = gk / G
+        fk = f[members][None, :]
+        dg[np.ix_(np.nonzero(U)[0], members)] = N_B / U.sum() * (fk - np.sum(fk * h, axis=1, keepdims=True)) / G
+    return scale * dg
 
 
 def bin_balance_grad_logits(z, topk_idx, expert_bin, n_bins, scale):

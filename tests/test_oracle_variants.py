@@ -160,3 +160,46 @@ def test_masked_bins_hold_only_chosen_experts():
     chosen_bins = eb[f["topk_idx"]]
     for j in range(X.shape[0]):
         assert set(np.nonzero(f["p"][j] > 0)[0]) == set(chosen_bins[j])
+
+
+def test_sigmoid_topk_weight_gradient_central_differences():
+    rng = np.random.default_rng(13)
+    z = rng.standard_normal((6, 9))
+    d = rng.standard_normal((6, 3))
+    idx = O.sigmoid_gate(z, None, k=3)["topk_idx"]
+
+    def L(zv):
+        s = O.sigmoid_gate(zv)["s"]
+        w = np.take_along_axis(s, idx.astype(np.int64), axis=1)
+        return float(np.sum(d * w / w.sum(axis=1, keepdims=True)))
+
+    grad = O.sigmoid_topk_weight_grad_logits(O.sigmoid_gate(z)["s"], idx, d)
+    h = 1e-6
+    num = np.zeros_like(z)
+    for i in np.ndindex(*z.shape):
+        zp, zm = z.copy(), z.copy()
+        zp[i] += h
+        zm[i] -= h
+        num[i] = (L(zp) - L(zm)) / (2 * h)
+    np.testing.assert_allclose(grad, num, rtol=1e-6, atol=1e-9)
+
+
+def test_balance_gradient_at_the_gate_central_differences():
+    # dL/dg from bin_balance_grad_gate against differences of eq. (16) in g itself (f held at the
+    # counts of the fixed choice), and the logits form through the softmax Jacobian
+    rng = np.random.default_rng(14)
+    z = rng.standard_normal((12, 8))
+    g = O.softmax_gate(z)
+    idx, _ = O.topk_route(z, g, 3)
+    eb = np.arange(8) // 2
+    dg = O.bin_balance_grad_gate(g, idx, eb, 4, 1.0)
+    h = 1e-7
+    num = np.zeros_like(g)
+    for i in np.ndindex(*g.shape):
+        gp, gm = g.copy(), g.copy()
+        gp[i] += h
+        gm[i] -= h
+        num[i] = (O.bin_balance_loss(gp, idx, eb, 4)[0] - O.bin_balance_loss(gm, idx, eb, 4)[0]) / (2 * h)
+    np.testing.assert_allclose(dg, num, rtol=1e-5, atol=1e-8)
+    np.testing.assert_allclose(O.softmax_grad_logits(g, dg), O.bin_balance_grad_logits(z, idx, eb, 4, 1.0),
+                               rtol=1e-12, atol=1e-15)
