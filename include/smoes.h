@@ -54,6 +54,8 @@ typedef enum {
   SMOES_SCORE_GMM = 3             /* Gaussian-mixture estimator (supplementary)     */
 } smoes_score_mode;
 
+typedef enum { SMOES_GATE_SOFTMAX = 0, SMOES_GATE_SIGMOID = 1 } smoes_gate;
+
 typedef struct smoes_plan_s* smoes_plan;
 
 /* Shape and routing metadata of one router layer (Secs. 3.1, 3.3).
@@ -67,6 +69,15 @@ typedef struct smoes_plan_s* smoes_plan;
  *   renorm_topk: 0 -> top-k weights are the softmax scores; 1 -> renormalised over the top-k.
  *   attn_max_heads: largest head count passed to smoes_modality_score(SMOES_SCORE_ATTN)
  *   (sizes the per-head partial sums in the workspace); 0 if the attention score is not used.
+ *   gate: SMOES_GATE_SOFTMAX (Sec. 3.1) or SMOES_GATE_SIGMOID (the sigmoid router with a
+ *   selection bias of the paper's backbone table: affinities s = sigmoid(z), experts chosen by
+ *   the top-k of s + score_bias, top-k weights s / sum of the chosen s (always renormalised), and
+ *   the g of eq. (12) read as s / sum_e s).
+ *   score_bias: device array [E] float32 read by every forward of a SMOES_GATE_SIGMOID plan (the
+ *   caller may update it in place between steps), or NULL for no bias.
+ *   mi_topk_mask: 0 -> the g summed into the bins of eq. (12) is the dense gate; 1 -> it is the
+ *   gate restricted to the chosen experts and renormalised over them (a reading the paper leaves
+ *   open). bin_prob then reports these masked bin sums.
  * Both host arrays are copied; the caller may free them after smoes_plan_create returns. */
 typedef struct {
   int T, d, E, k, n_bins, n_samples;
@@ -75,6 +86,9 @@ typedef struct {
   const int32_t* expert_bin_host;
   int renorm_topk;
   int attn_max_heads;
+  int gate;                            /* smoes_gate                                           */
+  const float* score_bias;
+  int mi_topk_mask;
 } smoes_router_desc;
 
 /* Gaussian-statistics score inputs, eqs. (8)-(9).

@@ -24,6 +24,7 @@ STATUS_NAMES = {0: "SMOES_OK", -1: "SMOES_ERR_INVALID_ARG", -2: "SMOES_ERR_UNSUP
                 -3: "SMOES_ERR_ALIGNMENT", -4: "SMOES_ERR_WORKSPACE", -5: "SMOES_ERR_CUDA",
                 -6: "SMOES_ERR_DEVICE_TIMEOUT", -7: "SMOES_ERR_DATA"}
 SMOES_F32, SMOES_BF16 = 0, 1
+SMOES_GATE_SOFTMAX, SMOES_GATE_SIGMOID = 0, 1
 SMOES_SCORE_PROVIDED, SMOES_SCORE_GAUSS, SMOES_SCORE_ATTN, SMOES_SCORE_GMM = 0, 1, 2, 3
 
 
@@ -38,7 +39,8 @@ class RouterDesc(C.Structure):
                 ("n_bins", C.c_int), ("n_samples", C.c_int), ("dtype", C.c_int),
                 ("sample_offsets_host", C.POINTER(C.c_int32)),
                 ("expert_bin_host", C.POINTER(C.c_int32)), ("renorm_topk", C.c_int),
-                ("attn_max_heads", C.c_int)]
+                ("attn_max_heads", C.c_int), ("gate", C.c_int), ("score_bias", C.c_void_p),
+                ("mi_topk_mask", C.c_int)]
 
 
 class GaussArgs(C.Structure):
@@ -114,13 +116,14 @@ def smoes_status_string(code: int) -> str:
 
 
 def smoes_plan_create(T, d, E, k, n_bins, sample_offsets, expert_bin, dtype, renorm_topk=0,
-                      attn_max_heads=0):
+                      attn_max_heads=0, gate=0, score_bias=None, mi_topk_mask=0):
     """Returns (status, plan handle). sample_offsets [B+1] and expert_bin [E] are host arrays."""
     offs = np.ascontiguousarray(np.asarray(sample_offsets, dtype=np.int32))
     eb = np.ascontiguousarray(np.asarray(expert_bin, dtype=np.int32))
     desc = RouterDesc(T, d, E, k, n_bins, max(len(offs) - 1, 0), dtype,
                       offs.ctypes.data_as(C.POINTER(C.c_int32)),
-                      eb.ctypes.data_as(C.POINTER(C.c_int32)), renorm_topk, attn_max_heads)
+                      eb.ctypes.data_as(C.POINTER(C.c_int32)), renorm_topk, attn_max_heads,
+                      int(gate), _p(score_bias), int(mi_topk_mask))
     h = C.c_void_p()
     code = _lib.smoes_plan_create(C.byref(desc), C.byref(h))
     return code, h
@@ -246,9 +249,11 @@ class Router:
     """
 
     def __init__(self, T, d, E, k, n_bins, sample_offsets, expert_bin, dtype=SMOES_BF16,
-                 renorm_topk=0, attn_max_heads=0, device="cuda"):
+                 renorm_topk=0, attn_max_heads=0, device="cuda", gate=0, score_bias=None,
+                 mi_topk_mask=0):
         code, self.plan = smoes_plan_create(T, d, E, k, n_bins, sample_offsets, expert_bin, dtype,
-                                            renorm_topk, attn_max_heads)
+                                            renorm_topk, attn_max_heads, gate, score_bias,
+                                            mi_topk_mask)
         _check(code, "smoes_plan_create")
         self.T, self.d, self.E, self.k, self.K = T, d, E, k, n_bins
         self.B = len(sample_offsets) - 1

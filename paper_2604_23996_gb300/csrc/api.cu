@@ -96,7 +96,9 @@ Dims make_dims(const smoes_plan_s* P) {
   m.K = d.n_bins;
   m.B = d.n_samples;
   m.N_B = P->N_B;
-  m.renorm = d.renorm_topk ? 1 : 0;
+  m.renorm = (d.renorm_topk || d.gate == SMOES_GATE_SIGMOID) ? 1 : 0;
+  m.gate = d.gate == SMOES_GATE_SIGMOID ? 1 : 0;
+  m.mask = d.mi_topk_mask ? 1 : 0;
   m.pstride = piece_stride(d.n_bins);
   m.n_groups = P->n_groups;
   m.contig_bins = P->contig_bins ? 1 : 0;
@@ -194,6 +196,7 @@ smoes_status router_fwd(smoes_plan P, const void* X, const void* W, const float*
   p.X = X;
   p.W = W;
   p.M_in = M_in;
+  p.score_bias = d.score_bias;
   p.mu = gauss ? gauss->mu : nullptr;
   p.var = gauss ? gauss->var : nullptr;
   p.inv_tau = gauss ? 1.f / (gauss->tau > 0.f ? gauss->tau : 0.5f * d.d) : 1.f;
@@ -253,6 +256,9 @@ smoes_status smoes_plan_create(const smoes_router_desc* desc, smoes_plan* out) {
   if (d.T < 0 || d.d < 8 || d.d % 8 != 0 || d.E < 1 || d.k < 1 || d.n_bins < 1)
     return SMOES_ERR_INVALID_ARG;
   if (d.dtype != SMOES_F32 && d.dtype != SMOES_BF16) return SMOES_ERR_INVALID_ARG;
+  if (d.gate != SMOES_GATE_SOFTMAX && d.gate != SMOES_GATE_SIGMOID) return SMOES_ERR_INVALID_ARG;
+  if (d.mi_topk_mask != 0 && d.mi_topk_mask != 1) return SMOES_ERR_INVALID_ARG;
+  if (d.score_bias && (d.gate != SMOES_GATE_SIGMOID || !aligned16(d.score_bias))) return SMOES_ERR_INVALID_ARG;
   if (d.k > d.E || d.E % d.n_bins != 0) return SMOES_ERR_INVALID_ARG;
   if (d.E > kMaxExperts || d.k > kMaxTopK || d.n_bins > kMaxBins || d.E / d.n_bins > 32)
     return SMOES_ERR_UNSUPPORTED;
@@ -582,7 +588,7 @@ smoes_status smoes_router_bwd(smoes_plan P, const void* X, const void* W, const 
     return cuda_status(cudaMemsetAsync(dW, 0, sizeof(float) * static_cast<size_t>(d.E) * d.d, stream));
   }
   if (!X || !W || !M) return SMOES_ERR_INVALID_ARG;
-  if (d_topk_w && !topk_idx) return SMOES_ERR_INVALID_ARG;
+  if ((d_topk_w || d.mi_topk_mask) && !topk_idx) return SMOES_ERR_INVALID_ARG;
   if (!aligned16(X) || !aligned16(W) || !aligned16(M) || !aligned16(dW) || (dX && !aligned16(dX)))
     return SMOES_ERR_ALIGNMENT;
   if (d.dtype == SMOES_BF16 && d.E > 128) return SMOES_ERR_UNSUPPORTED;

@@ -86,13 +86,14 @@ __device__ __forceinline__ float upstream_at(const Upstream& u, int k, int e) {
 }
 
 // Gradient of the bin-level balance loss (eq. 16) at one token's logits, added to dz[N] of the
-// thread's N experts (g: their softmax scores, be: their bins (-1: none), fe: their f_e): for every
-// bin k the token routes to, dz_e += a_k h_e (f_e - sum_{e' in B_k} f_e' h_e') with h = g / (bin
-// sum). The bin sums run over the token's GS-lane thread group (xor shuffles); every lane takes
+// thread's N experts (g: their gate values, be: their bins (-1: none), fe: their f_e, fac: the
+// gate's own factor, 1 for the softmax and 1 - s for the sigmoid): for every bin k the token
+// routes to, dz_e += a_k h_e (f_e - sum_{e' in B_k} f_e' h_e') fac_e with h = g / (bin sum). The bin sums run over the token's GS-lane thread group (xor shuffles); every lane takes
 // the same k iterations, and a bin repeated among the token's selections adds nothing again.
 template <int GS, int N>
 __device__ __forceinline__ void add_balance_grad(const BwdParams& p, int j, bool valid, const float (&g)[N],
-                                                 const int (&be)[N], const float (&fe)[N], float (&dz)[N]) {
+                                                 const int (&be)[N], const float (&fe)[N],
+                                                 const float (&fac)[N], float (&dz)[N]) {
   const int k = p.dm.k;
   int seen[kMaxTopK];
 #pragma unroll
@@ -120,8 +121,52 @@ __device__ __forceinline__ void add_balance_grad(const BwdParams& p, int j, bool
       const float a = __ldg(p.ws.bal_a + bs), iv = 1.f / v, phi = w * iv;
 #pragma unroll
       for (int i = 0; i < N; ++i)
-        if (be[i] == bs) dz[i] = fmaf(a * g[i] * iv, fe[i] - phi, dz[i]);
+        if (be[i] == bs) dz[i] = fmaf(a * g[i] * iv * fac[i], fe[i] - phi, dz[i]);
     }
+  }
+}
+
+// MI gradient at one token's logits for the thread's N experts (a GS-lane group holds the token):
+//   dz_e = scale fac_e w_e (u_e - sum_e' w_e' u_e'),
+// with w the gate values that enter eq. (12) (the dense gate g, or with the top-k mask g on the
+// chosen experts renormalised over them) and fac_e = 1 (softmax) or 1 - s_e (sigmoid: through
+// g = s / sum s, s = sigmoid(z)). raw: the saved exp(z - max) or s; g = raw / sum raw.
+template <int GS, int N, bool kVar = true>
+__device__ __forceinline__ void mi_grad(const BwdParams& p, int j, bool valid, const int (&eidx)[N],
+                                        const float (&raw)[N], const float (&g)[N], const float (&u)[N],
+                                        float (&fac)[N], float (&dz)[N]) {
+  const Dims& dm = p.dm;
+  const bool gate = kVar && dm.gate, mask = kVar && dm.mask;   // kVar false: the softmax router
+  float w[N];
+#pragma unroll
+  for (int i = 0; i < N; ++i) w[i] = g[i];
+  if (mask) {
+    bool sel[N];
+#pragma unroll
+    for (int i = 0; i < N; ++i) sel[i] = false;
+    for (int s = 0; s < dm.k; ++s) {
+      const int es = valid ? __ldg(p.topk_idx + static_cast<size_t>(j) * dm.k + s) : -1;
+#pragma unroll
+      for (int i = 0; i < N; ++i) sel[i] = sel[i] || (eidx[i] == es);
+    }
+    float G = 0.f;
+#pragma unroll
+    for (int i = 0; i < N; ++i) G += sel[i] ? g[i] : 0.f;
+#pragma unroll
+    for (int o = 1; o < GS; o <<= 1) G += __shfl_xor_sync(0xffffffffu, G, o);
+    const float iG = G > 0.f ? 1.f / G : 0.f;
+#pragma unroll
+    for (int i = 0; i < N; ++i) w[i] = sel[i] ? g[i] * iG : 0.f;
+  }
+  float part = 0.f;
+#pragma unroll
+  for (int i = 0; i < N; ++i) part = fmaf(w[i], u[i], part);
+#pragma unroll
+  for (int o = 1; o < GS; o <<= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+#pragma unroll
+  for (int i = 0; i < N; ++i) {
+    fac[i] = gate ? 1.f - raw[i] : 1.f;
+    dz[i] = p.scale * fac[i] * w[i] * (u[i] - part);
   }
 }
 
@@ -138,7 +183,7 @@ __device__ __forceinline__ void add_balance_grad(const BwdParams& p, int j, bool
 // register budget otherwise).
 constexpr int kDzRep = 2;
 
-template <int TPT, bool kUp, bool kBal>
+template <int TPT, bool kUp, bool kBal, bool kVar>
 __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
   pdl_wait();                                         // scores and tables of the forward
   pdl_trigger();
@@ -202,10 +247,10 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
 #pragma unroll
   for (int q = 0; q < kDzRep; ++q) {
     if (j[q] >= n_rows) continue;                     // whole TPT groups skip together
-    float g[8] = {ga[q].x, ga[q].y, ga[q].z, ga[q].w, gb[q].x, gb[q].y, gb[q].z, gb[q].w};
-    float u[8];
+    const float raw[8] = {ga[q].x, ga[q].y, ga[q].z, ga[q].w, gb[q].x, gb[q].y, gb[q].z, gb[q].w};
+    float g[8], u[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) { g[i] *= ginv[q]; u[i] = 0.f; }        // the softmax score g_je
+    for (int i = 0; i < 8; ++i) { g[i] = raw[i] * ginv[q]; u[i] = 0.f; }   // the gate value g_je
     if (valid[q]) {
       const float dv = m[q].x - 0.5f, dt = m[q].y - 0.5f;
       // the sample's coefficient table was written by the forward kernel and is read-only here
@@ -226,22 +271,21 @@ __global__ void __launch_bounds__(256) k_dz_prep(const BwdParams p) {
         }
       }
     }
-    float part = 0.f;
+    int eidx[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) part = fmaf(g[i], u[i], part);
-#pragma unroll
-    for (int o = 1; o < TPT; o <<= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-    float dz[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) dz[i] = p.scale * g[i] * (u[i] - part);
+    for (int i = 0; i < 8; ++i) eidx[i] = e0 + i < E ? e0 + i : -2;
+    float dz[8], fac[8];
+    mi_grad<TPT, 8, kVar>(p, j[q], valid[q], eidx, raw, g, u, fac, dz);
     if (kUp && valid[q]) {
       Upstream up;
       load_upstream(p, j[q], up);
 #pragma unroll
       for (int i = 0; i < 8; ++i)
-        if (e0 + i < E) dz[i] += g[i] * (upstream_at(up, k, e0 + i) - up.gdt);
+        if (e0 + i < E)
+          dz[i] += (kVar && dm.gate) ? fac[i] * g[i] * upstream_at(up, k, e0 + i)   // diagonal
+                                     : g[i] * (upstream_at(up, k, e0 + i) - up.gdt);
     }
-    if (kBal && bal) add_balance_grad<TPT, 8>(p, j[q], valid[q], g, be, fe, dz);
+    if (kBal && bal) add_balance_grad<TPT, 8>(p, j[q], valid[q], g, be, fe, fac, dz);
     if (valid[q] && p.dlogits) {
       float* dl = p.dlogits + static_cast<size_t>(j[q]) * E;
       if (vec) {
@@ -590,41 +634,32 @@ k_router_bwd_f32(const BwdParams p) {
     if (has_up) load_upstream(p, j, up);
     const float* g = p.ws.gsave + static_cast<size_t>(valid ? j : 0) * E;
     const float ginv = valid ? p.ws.ginv[j] : 0.f;
-    float part = 0.f;
-    for (int e = qd; e < E; e += 4) {
-      if (valid) {
-        const int b = p.ws.expert_bin[e];
-        part += g[e] * ginv * (tb[2 * K + b] + dv * tb[b] + dt * tb[K + b]);
-      }
-    }
-    part += __shfl_xor_sync(0xffffffffu, part, 1);
-    part += __shfl_xor_sync(0xffffffffu, part, 2);
-    float dzv[EB / 4];
+    // the token's 4-thread group holds experts qd, qd + 4, ...
+    constexpr int NQ = EB / 4;
+    int eidx[NQ], bq[NQ];
+    float raw[NQ], gq[NQ], uq[NQ], fq[NQ], fac[NQ], dzv[NQ];
 #pragma unroll
-    for (int i = 0; i < EB / 4; ++i) {
+    for (int i = 0; i < NQ; ++i) {
       const int e = qd + 4 * i;
-      float v = 0.f;
-      if (valid && e < E) {
-        const int b = p.ws.expert_bin[e];
-        const float u = tb[2 * K + b] + dv * tb[b] + dt * tb[K + b];
-        const float ge = g[e] * ginv;
-        v = p.scale * ge * (u - part);
-        if (has_up) v += ge * (upstream_at(up, k, e) - up.gdt);
-      }
-      dzv[i] = v;
+      const bool in = valid && e < E;
+      eidx[i] = e < E ? e : -2;
+      bq[i] = in ? p.ws.expert_bin[e] : -1;
+      raw[i] = in ? g[e] : 0.f;
+      gq[i] = raw[i] * ginv;
+      uq[i] = in ? tb[2 * K + bq[i]] + dv * tb[bq[i]] + dt * tb[K + bq[i]] : 0.f;
+    }
+    mi_grad<4, NQ>(p, j, valid, eidx, raw, gq, uq, fac, dzv);
+    if (has_up) {
+#pragma unroll
+      for (int i = 0; i < NQ; ++i)
+        if (eidx[i] >= 0)
+          dzv[i] += dm.gate ? fac[i] * gq[i] * upstream_at(up, k, eidx[i])
+                            : gq[i] * (upstream_at(up, k, eidx[i]) - up.gdt);
     }
     if (p.topk_idx && __ldcg(p.ws.bal_flag) != 0u) {   // the balance term (eq. 16); block-uniform
-      float gq[EB / 4], fq[EB / 4];
-      int bq[EB / 4];
 #pragma unroll
-      for (int i = 0; i < EB / 4; ++i) {
-        const int e = qd + 4 * i;
-        const bool in = valid && e < E;
-        gq[i] = in ? g[e] * ginv : 0.f;
-        bq[i] = in ? p.ws.expert_bin[e] : -1;
-        fq[i] = in ? p.ws.bal_f[e] : 0.f;
-      }
-      add_balance_grad<4, EB / 4>(p, j, valid, gq, bq, fq, dzv);
+      for (int i = 0; i < NQ; ++i) fq[i] = bq[i] >= 0 ? p.ws.bal_f[eidx[i]] : 0.f;
+      add_balance_grad<4, NQ>(p, j, valid, gq, bq, fq, fac, dzv);
     }
 #pragma unroll
     for (int i = 0; i < EB / 4; ++i) {
@@ -759,10 +794,14 @@ cudaError_t launch_dz_prep(const BwdParams& p, cudaStream_t s) {
   // the upstream-gradient and balance variants keep their tables out of the common kernel's
   // registers; the balance variant still checks the arming flag on the device
   const bool up = p.d_topk_w != nullptr, bal = p.balance_armed != 0;
+  const bool var = p.dm.gate != 0 || p.dm.mask != 0;      // sigmoid gate or top-k-masked g
   auto pick = [&](auto tpt) {
     constexpr int TPT = decltype(tpt)::value;
-    return up ? (bal ? k_dz_prep<TPT, true, true> : k_dz_prep<TPT, true, false>)
-              : (bal ? k_dz_prep<TPT, false, true> : k_dz_prep<TPT, false, false>);
+    if (var)
+      return up ? (bal ? k_dz_prep<TPT, true, true, true> : k_dz_prep<TPT, true, false, true>)
+                : (bal ? k_dz_prep<TPT, false, true, true> : k_dz_prep<TPT, false, false, true>);
+    return up ? (bal ? k_dz_prep<TPT, true, true, false> : k_dz_prep<TPT, true, false, false>)
+              : (bal ? k_dz_prep<TPT, false, true, false> : k_dz_prep<TPT, false, false, false>);
   };
   if (E_pad == 64) return launch_pdl(pick(std::integral_constant<int, 8>()), dim3(blocks), dim3(256), 0, s, p);
   if (E_pad == 128) return launch_pdl(pick(std::integral_constant<int, 16>()), dim3(blocks), dim3(256), 0, s, p);

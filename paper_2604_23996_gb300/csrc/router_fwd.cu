@@ -354,16 +354,35 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
 #pragma unroll
   for (int i = 0; i < KM; ++i) tk[i] = tk2[i] = -CUDART_INF_F;
   float mx = -CUDART_INF_F, mx2 = -CUDART_INF_F;
+  if (!dm.gate) {
 #pragma unroll 1
-  for (int c = cb; c < ce; ++c) {
-    float v[16];
-    src.load16(c, v);
+    for (int c = cb; c < ce; ++c) {
+      float v[16];
+      src.load16(c, v);
 #pragma unroll
-    for (int t = 0; t < 16; t += 2) {
-      mx = fmaxf(mx, v[t]);
-      mx2 = fmaxf(mx2, v[t + 1]);
-      topk_push<KM>(tk, topk_key(v[t], c * 16 + t, imask));
-      topk_push<KM>(tk2, topk_key(v[t + 1], c * 16 + t + 1, imask));
+      for (int t = 0; t < 16; t += 2) {
+        mx = fmaxf(mx, v[t]);
+        mx2 = fmaxf(mx2, v[t + 1]);
+        topk_push<KM>(tk, topk_key(v[t], c * 16 + t, imask));
+        topk_push<KM>(tk2, topk_key(v[t + 1], c * 16 + t + 1, imask));
+      }
+    }
+  } else {                           // sigmoid gate: the choice ranks s + bias (padding stays last)
+#pragma unroll 1
+    for (int c = cb; c < ce; ++c) {
+      float v[16];
+      src.load16(c, v);
+#pragma unroll
+      for (int t = 0; t < 16; ++t) {
+        const int e = c * 16 + t;
+        mx = fmaxf(mx, v[t]);
+        v[t] = e < E ? sigmoid_acc(v[t]) + (p.score_bias ? __ldg(p.score_bias + e) : 0.f) : -FLT_MAX;
+      }
+#pragma unroll
+      for (int t = 0; t < 16; t += 2) {
+        topk_push<KM>(tk, topk_key(v[t], c * 16 + t, imask));
+        topk_push<KM>(tk2, topk_key(v[t + 1], c * 16 + t + 1, imask));
+      }
     }
   }
   mx = fmaxf(mx, mx2);
@@ -398,10 +417,18 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
     float v[16];
     src.load16(c, v);
     float ps[4] = {0.f, 0.f, 0.f, 0.f};
+    if (!dm.gate) {
 #pragma unroll
-    for (int t = 0; t < 16; ++t) {
-      v[t] = exp2f(fmaf(v[t], kLog2e, -mxl));
-      ps[t & 3] += v[t];
+      for (int t = 0; t < 16; ++t) {
+        v[t] = exp2f(fmaf(v[t], kLog2e, -mxl));                 // saved e = exp(z - max)
+        ps[t & 3] += v[t];
+      }
+    } else {
+#pragma unroll
+      for (int t = 0; t < 16; ++t) {
+        v[t] = sigmoid_acc(v[t]);                               // saved s = sigmoid(z)
+        ps[t & 3] += v[t];
+      }
     }
     sum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
     if (stg) {
@@ -460,7 +487,8 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
   // this group's bins (all of them for group 0 without a split): e sums -> probabilities
   const int kb0 = split && grp ? 16 * nc0 / dm.N_B : 0;
   const int kb1 = split && !grp ? 16 * nc0 / dm.N_B : (grp && !split ? 0 : K);
-  for (int b = kb0; b < kb1; ++b) prow[b * kPsStride] = valid ? prow[b * kPsStride] * inv : 0.f;
+  if (!dm.mask)                   // (the top-k-masked bins are written by group 0 below)
+    for (int b = kb0; b < kb1; ++b) prow[b * kPsStride] = valid ? prow[b * kPsStride] * inv : 0.f;
 
   float Mv = 0.f, Mt = 0.f, dv = 0.f, dt = 0.f;
   if (grp == 0) {
@@ -478,6 +506,9 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
             const uint32_t e = static_cast<uint32_t>(topk_index(tk[i], imask));
             const uint32_t qd = ((e & 31u) >> 2) ^ static_cast<uint32_t>(row & 7);
             w[i] = *reinterpret_cast<const float*>(es.stg + (e >> 5) * 16384u + row * 128 + (qd << 4) + (e & 3u) * 4u) * inv;
+          } else if (dm.gate) {      // s from the key s + bias (renormalised below)
+            const int e = topk_index(tk[i], imask);
+            w[i] = topk_logit(tk[i], imask) - (p.score_bias ? __ldg(p.score_bias + e) : 0.f);
           } else {
             w[i] = exp2f(fmaf(topk_logit(tk[i], imask), kLog2e, -mxl)) * inv;
           }
@@ -494,6 +525,20 @@ __device__ void epilogue_tile(const FwdParams& p, const Src& src, const Release&
           tw[i] = w[i] * wsc;
         }
       }
+      if (dm.mask) {                 // eq. (12) on the gate restricted to the top-k, renormalised
+        for (int b = 0; b < K; ++b) prow[b * kPsStride] = 0.f;
+        const float iw = 1.f / wsum;
+#pragma unroll
+        for (int i = 0; i < KM; ++i) {
+          if (i < k) {
+            const int e = topk_index(tk[i], imask);
+            const int b = dm.contig_bins ? e / dm.N_B : __ldg(p.ws.expert_bin + e);
+            prow[b * kPsStride] += w[i] * iw;
+          }
+        }
+      }
+    } else if (dm.mask) {
+      for (int b = 0; b < K; ++b) prow[b * kPsStride] = 0.f;
     }
     if (p.perm.perm_token) {         // (token, bin) pairs of this warp's rows, per bin
       uint32_t bins = 0u;

@@ -61,6 +61,8 @@ struct WsView {
 
 struct Dims {
   int T, d, E, k, K, B, N_B, renorm;
+  int gate;                  // 0 softmax, 1 sigmoid (affinities s; g = s / sum s; renorm forced)
+  int mask;                  // 1: the g of eq. (12) is restricted to the top-k and renormalised
   int pstride;               // piece_stride(K)
   int n_groups;              // ceil(T / 128): forward tiles = partial-sum groups
   int contig_bins;           // bin b holds experts [b N_B, (b+1) N_B) and N_B % 4 == 0
@@ -86,6 +88,7 @@ struct FwdParams {
   const void* X;
   const void* W;             // [E, d] (read directly by the fp32 path; bf16 goes through TMA)
   const float* M_in;         // provided scores, or null when the Gaussian score is fused
+  const float* score_bias;   // [E] selection bias of the sigmoid gate, or null
   const float* mu;           // [2, d] (Gaussian mode)
   const float* var;          // [2, d]
   float inv_tau;
