@@ -185,6 +185,20 @@ smoes_status smoes_modality_score(smoes_plan plan, smoes_score_mode mode,
                                   const smoes_score_args* args, float* M,
                                   void* ws, size_t ws_bytes, cudaStream_t stream);
 
+/* (1b) Causal attention forward that also yields the attention-accumulated score (Sec. 3.2.1,
+ *   eqs. (2)-(4); the form the paper's supplementary gives for FlashAttention-style kernels: the
+ *   carried score is one more value column). args as for SMOES_SCORE_ATTN (Q [B, H, S, hd], K with
+ *   n_kv_heads heads [B, n_kv_heads, S, hd], bf16); V [B, n_kv_heads, S, hd] bf16; grouped-query
+ *   heads: query head h reads key/value head h / (H / n_kv_heads) (H % n_kv_heads == 0).
+ *   Outputs: O [B, H, S, hd] bf16 = softmax(sm_scale Q K^T + key_bias) V per head (the softmax
+ *   weights pass to the tensor cores in bf16, as in FlashAttention), and M [T, 2] as for
+ *   smoes_modality_score(SMOES_SCORE_ATTN) (the head-averaged vision mass, optionally blended
+ *   by eq. (4)). Requires hd == 128 and S % 128 == 0 (else SMOES_ERR_UNSUPPORTED); key_bias,
+ *   is_vision and m_prev 16-byte aligned; H <= attn_max_heads of the plan. */
+smoes_status smoes_attention_fwd(smoes_plan plan, const smoes_attn_args* args, const void* V,
+                                 int n_kv_heads, void* O, float* M, void* ws, size_t ws_bytes,
+                                 cudaStream_t stream);
+
 /* (2) Router forward with the MI regulariser (Secs. 3.1, 3.3, 3.4).
  *   X [T, d], W [E, d] (plan dtype). Scores: M_in [T, 2] (SMOES_SCORE_PROVIDED, gauss == NULL),
  *   or gauss != NULL (fused Gaussian score; gauss->X is ignored, X is used) and the scores are

@@ -85,6 +85,7 @@ _sig = {
                                          _sz, _vp]),
     "smoes_adaptive_bins": (_i, [_vp, _vp, C.c_double, _vp, _vp, _vp, _vp]),
     "smoes_bin_balance": (_i, [_vp, _vp, _f, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "smoes_attention_fwd": (_i, [_vp, C.POINTER(AttnArgs), _vp, _i, _vp, _vp, _vp, _sz, _vp]),
 }
 for _name, (_res, _args) in _sig.items():
     _fn = getattr(_lib, _name)
@@ -227,6 +228,19 @@ def smoes_gaussian_stats_update(plan, X, is_vision, beta, N, S_mu, S_var, mu, va
     return _lib.smoes_gaussian_stats_update(plan, _p(X), _p(is_vision), float(beta), _p(N), _p(S_mu),
                                             _p(S_var), _p(mu), _p(var), _p(ws),
                                             ws.numel() * ws.element_size(), _stream(stream))
+
+
+def _attn_args(a):
+    return AttnArgs(_p(a["Q"]), _p(a["K"]), a["B"], a["H"], a["S"], a["hd"], _p(a.get("is_vision")),
+                    _p(a.get("m_prev")), _p(a.get("key_bias")), float(a["sm_scale"]),
+                    int(a.get("causal", 1)), _p(a.get("xattn_norm")), _p(a.get("x_norm")))
+
+
+def smoes_attention_fwd(plan, attn, V, n_kv_heads, O, M, ws, stream=None) -> int:
+    """Attention forward with the vision score (O and M); attn as for smoes_modality_score."""
+    args = _attn_args(attn)
+    return _lib.smoes_attention_fwd(plan, C.byref(args), _p(V), int(n_kv_heads), _p(O), _p(M), _p(ws),
+                                    ws.numel() * ws.element_size(), _stream(stream))
 
 
 def smoes_bin_balance(plan, topk_idx, loss_scale, loss_bal, ws, f_e=None, P_e=None, stream=None) -> int:

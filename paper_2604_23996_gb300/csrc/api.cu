@@ -528,6 +528,60 @@ smoes_status smoes_modality_score(smoes_plan P, smoes_score_mode mode, const smo
   return SMOES_ERR_INVALID_ARG;
 }
 
+smoes_status smoes_attention_fwd(smoes_plan P, const smoes_attn_args* args, const void* V,
+                                 int n_kv_heads, void* O, float* M, void* ws, size_t ws_bytes,
+                                 cudaStream_t stream) {
+  if (!P || !args || !M || !O || !V) return SMOES_ERR_INVALID_ARG;
+  smoes_status st = check_ws(P, ws, ws_bytes);
+  if (st != SMOES_OK) return st;
+  const smoes_router_desc& d = P->desc;
+  const smoes_attn_args& a = *args;
+  if (!a.Q || !a.K || a.B < 1 || a.H < 1 || a.S < 1 || n_kv_heads < 1) return SMOES_ERR_INVALID_ARG;
+  if (static_cast<long long>(a.B) * a.S != d.T) return SMOES_ERR_INVALID_ARG;
+  if ((a.is_vision == nullptr) == (a.m_prev == nullptr)) return SMOES_ERR_INVALID_ARG;
+  if ((a.xattn_norm == nullptr) != (a.x_norm == nullptr)) return SMOES_ERR_INVALID_ARG;
+  if (a.H % n_kv_heads != 0) return SMOES_ERR_INVALID_ARG;
+  if (a.hd != 128 || a.S % 128 != 0) return SMOES_ERR_UNSUPPORTED;
+  if (a.H > d.attn_max_heads) return SMOES_ERR_WORKSPACE;
+  if (!aligned16(a.Q) || !aligned16(a.K) || !aligned16(V) || !aligned16(O) || !aligned16(M) ||
+      (a.key_bias && !aligned16(a.key_bias)) || (a.is_vision && !aligned16(a.is_vision)) ||
+      (a.m_prev && !aligned16(a.m_prev)))
+    return SMOES_ERR_ALIGNMENT;
+  WsView v = make_view(P, ws);
+  AttnFwdParams fp{};
+  AttnParams& p = fp.a;
+  p.B = a.B;
+  p.H = a.H;
+  p.S = a.S;
+  p.hd = a.hd;
+  p.T = d.T;
+  p.Q = a.Q;
+  p.K = a.K;
+  p.is_vision = a.is_vision;
+  p.m_prev = a.m_prev;
+  p.key_bias = a.key_bias;
+  p.scale_log2 = a.sm_scale * 1.4426950408889634f;
+  p.causal = a.causal ? 1 : 0;
+  p.xattn_norm = a.xattn_norm;
+  p.x_norm = a.x_norm;
+  p.M = M;
+  p.part = v.attn_part;
+  p.ticket = v.attn_ticket;
+  p.status = v.status;
+  p.n_qtiles = a.S / 128;
+  p.n_items = a.B * a.H * p.n_qtiles;
+  p.limit_ns = P->limit_ns;
+  fp.Hkv = n_kv_heads;
+  CUtensorMap tq, tk, tv, to;
+  const uint64_t rq = static_cast<uint64_t>(a.B) * a.H * a.S, rk = static_cast<uint64_t>(a.B) * n_kv_heads * a.S;
+  if (!encode_bf16_2d(&tq, a.Q, rq, a.hd, 128, 64, true) || !encode_bf16_2d(&tk, a.K, rk, a.hd, 128, 64, true) ||
+      !encode_bf16_2d(&tv, V, rk, a.hd, 128, 64, true) || !encode_bf16_2d(&to, O, rq, a.hd, 128, 64, true))
+    return SMOES_ERR_CUDA;
+  const cudaError_t e = launch_attn_fwd(fp, tq, tk, tv, to, P->n_sms, stream);
+  if (e == cudaErrorNotSupported) return SMOES_ERR_UNSUPPORTED;
+  return cuda_status(e);
+}
+
 smoes_status smoes_router_fwd(smoes_plan P, const void* X, const void* W, const float* M_in,
                               const smoes_gauss_args* gauss, float* M_out, int32_t* topk_idx,
                               float* topk_w, float* bin_prob, float* joint, float* mi, float* loss,

@@ -305,6 +305,15 @@ cudaError_t launch_gauss_coef(const float* mu, const float* var, int d, int dcoe
 cudaError_t launch_stats_update(const StatsParams& p, bool bf16, cudaStream_t s);
 cudaError_t launch_adaptive_bins(const BinsParams& p, cudaStream_t s);
 cudaError_t launch_bin_balance(const BalParams& p, cudaStream_t s);
+// Attention forward with the vision score as one more value column (eqs. 2-4), grouped-query
+// heads: K and V have Hkv heads, query head h reads key/value head h / (H / Hkv). O [B, H, S, hd]
+// bf16 (written through the TMA map), M as for the mass-only kernel.
+struct AttnFwdParams {
+  AttnParams a;
+  int Hkv;
+};
+cudaError_t launch_attn_fwd(const AttnFwdParams& p, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+                            const CUtensorMap& tmV, const CUtensorMap& tmO, int n_sms, cudaStream_t s);
 cudaError_t launch_gmm_score(const GmmParams& p, smoes_dtype dt, int n_sms, cudaStream_t s);
 cudaError_t launch_attn_mass(const AttnParams& p, const CUtensorMap& tmQ, const CUtensorMap& tmK,
                              int n_sms, cudaStream_t s);
