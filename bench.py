@@ -53,12 +53,15 @@ def parse(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-sweep", action="store_true")
+    ap.add_argument("--no-next", action="store_true",
+                    help="skip the timings of the next rows' kernels (statistics, binning, "
+                         "balance, GMM score, attention forward)")
     ap.add_argument("--profile", action="store_true",
                     help="short run for ncu: no clock load window, no e2e, no CPU baseline, no sweep")
     ap.add_argument("--oracle-child", default=None, help=argparse.SUPPRESS)
     args = ap.parse_args(argv)
     if args.profile:
-        args.no_e2e = args.no_cpu_baseline = args.no_sweep = True
+        args.no_e2e = args.no_cpu_baseline = args.no_sweep = args.no_next = True
     return args
 
 
@@ -591,6 +594,101 @@ def run_e2e(st, args, world, dev, rate_of):
             "note": "inputs of step i+1 copied while step i computes (two device buffers)"}
 
 
+def graph_time(fn, steps, flush):
+    """Mean device time (ms) of fn replayed from a CUDA graph, L2 flushed before each replay."""
+    import torch
+    fn()
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            fn()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    for _ in range(3):
+        g.replay()
+    ts = []
+    for _ in range(steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        g.replay()
+        b.record()
+        b.synchronize()
+        ts.append(a.elapsed_time(b))
+    return float(np.mean(ts))
+
+
+def measure_next(bd, st, dev, flush, steps, hbm, tf_sus, sm_mhz, n_sms):
+    """Timings of the next rows' kernels beside the hot path (one layer's worth each), with their
+    rooflines: the Gaussian statistics update and the GMM score over this batch's X, the
+    bin-level balance loss over its saved softmax, the adaptive binning, and the attention
+    forward with the vision score on the attention workload (8 x 16 heads x 4096, hd 128), with
+    H_kv = 16 and with grouped-query heads (H_kv = 4)."""
+    import torch
+    from paper_2604_23996_gb300.workloads import attn_workload
+    wl, r = st.wl, st.r
+    T, d, E, k, K = wl.T, wl.d, wl.E, wl.k, wl.n_bins
+    b = wl.X.element_size()
+    out = {}
+
+    def hbm_entry(ms, by, kern):
+        ach = by / (ms * 1e-3) / 1e9
+        return {"us": 1e3 * ms, "bound": "hbm", "bytes": by, "achieved": ach, "peak": hbm,
+                "unit": "GB/s", "frac": ach / hbm, "kernel": kern}
+
+    N = torch.zeros(2, dtype=torch.float64, device=dev)
+    S_mu = torch.zeros((2, d), dtype=torch.float64, device=dev)
+    S_var = torch.zeros((2, d), dtype=torch.float64, device=dev)
+    mu, var = torch.empty((2, d), device=dev), torch.empty((2, d), device=dev)
+    ms = graph_time(lambda: bd.smoes_gaussian_stats_update(r.plan, st.X, st.is_vis, 0.99, N, S_mu, S_var,
+                                                           mu, var, r.ws), steps, flush)
+    out["gaussian_stats_update"] = hbm_entry(ms, T * d * b + T, "k_stats_partial + k_stats_finalize")
+    C_bar = torch.zeros((2, E), dtype=torch.float64, device=dev)
+    eb = torch.empty(E, dtype=torch.int32, device=dev)
+    st.fwd_perm()
+    ms = graph_time(lambda: bd.smoes_adaptive_bins(r.plan, r.expert_counts, 0.99, C_bar, eb), steps, flush)
+    out["adaptive_bins"] = {"us": 1e3 * ms, "bound": "latency", "kernel": "k_adaptive_bins (one block)"}
+    lb = torch.empty(1, device=dev)
+    ms = graph_time(lambda: bd.smoes_bin_balance(r.plan, r.topk_idx, 1e-3, lb, r.ws), steps, flush)
+    out["bin_balance"] = hbm_entry(ms, T * E * 4 + T * k * 4, "k_bal_partial + k_bal_finalize")
+    if wl.dtype == torch.bfloat16:
+        C = 2
+        lp = torch.log(torch.full((2, C), 0.5, device=dev))
+        mu2 = st.mu[:, None, :].repeat(1, C, 1).contiguous()
+        var2 = st.var[:, None, :].repeat(1, C, 1).contiguous()
+        Mg = torch.empty((T, 2), device=dev)
+        gmm = dict(X=st.X, n_components=C, log_pi=lp, mu=mu2, var=var2, tau=wl.tau)
+        ms = graph_time(lambda: bd.smoes_modality_score(r.plan, bd.SMOES_SCORE_GMM, Mg, r.ws, gmm=gmm),
+                        steps, flush)
+        out["gmm_score_2"] = hbm_entry(ms, T * d * b + 8 * T, "k_gmm_coef + k_gmm_score (2 components)")
+    aw = attn_workload()
+    Ta = aw.B * aw.S
+    ra = bd.Router(Ta, 64, 16, 2, 4, [0, Ta], np.arange(16) // 4, attn_max_heads=aw.H)
+    Ma = torch.empty((Ta, 2), device=dev)
+    Q = aw.Q.to(dev)
+    rng = np.random.default_rng(11)
+    for hkv in (aw.H, aw.H // 4):
+        Kt = aw.K.to(dev) if hkv == aw.H else aw.K[:, :hkv].contiguous().to(dev)
+        V = torch.from_numpy(rng.standard_normal((aw.B, hkv, aw.S, aw.hd), dtype=np.float32)).to(torch.bfloat16).to(dev)
+        Oo = torch.empty((aw.B, aw.H, aw.S, aw.hd), dtype=torch.bfloat16, device=dev)
+        attn = dict(Q=Q, K=Kt, B=aw.B, H=aw.H, S=aw.S, hd=aw.hd, sm_scale=aw.sm_scale, causal=1,
+                    key_bias=torch.from_numpy(aw.key_bias).to(dev), is_vision=torch.from_numpy(aw.is_vision).to(dev))
+        ms = graph_time(lambda: bd.smoes_attention_fwd(ra.plan, attn, V, hkv, Oo, Ma, ra.ws), steps, flush)
+        pairs = float(aw.B) * aw.H * aw.S * (aw.S + 1) / 2.0
+        flops = 4.0 * pairs * aw.hd                            # causal Q K^T and P V
+        ach = flops / (ms * 1e-3) / 1e12
+        exp_peak = 16 * n_sms * sm_mhz * 1e-3                  # Gexp/s on the special-function unit
+        out[f"attention_fwd_hkv{hkv}"] = {
+            "us": 1e3 * ms, "bound": "tensor", "flops": flops, "achieved": ach, "peak": tf_sus,
+            "unit": "TFLOP/s", "frac": ach / tf_sus, "exp_rate_frac": pairs / (ms * 1e-3) / 1e9 / exp_peak,
+            "kernel": "k_attn_fwd (8x16x4096, hd 128, causal)"}
+        del V, Oo, Kt
+    return out
+
+
 def main():
     args = parse()
     if args.oracle_child:
@@ -672,6 +770,11 @@ def main():
                              "step_frac": t_roof / (ms * 1e-3)}
 
     e2e = None if args.no_e2e else run_e2e(st, args, world, dev, lambda ms: job_rate(wl.T, world, ms))
+    nxt = None
+    if not args.no_next and rank == 0 and args.config == DEFAULT_CONFIG and args.tokens is None:
+        nxt = measure_next(bd, st, dev, flush, args.steps, peaks()[0], peaks()[2],
+                           float(clk.get("sm_max_mhz") or 2070.0),
+                           torch.cuda.get_device_properties(dev).multi_processor_count)
 
     if rank != 0:
         if world > 1:
@@ -730,6 +833,8 @@ def main():
     }
     if sweep is not None:
         line["sweep"] = sweep
+    if nxt is not None:
+        line["next_rows"] = nxt
     if not args.no_cpu_baseline and world == 1:
         rate, n, ntok, secs = cpu_oracle_rate(wl)
         one = single_thread_oracle_rate(wl)

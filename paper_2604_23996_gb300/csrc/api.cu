@@ -464,8 +464,8 @@ smoes_status smoes_modality_score(smoes_plan P, smoes_score_mode mode, const smo
     if (!g.X || !g.log_pi || !g.mu || !g.var) return SMOES_ERR_INVALID_ARG;
     if (g.n_components < 1) return SMOES_ERR_INVALID_ARG;
     if (g.n_components > kGmmMaxComponents) return SMOES_ERR_UNSUPPORTED;
-    // the forms' coefficients stay in shared memory: 2 (2C - 1) round_up(d, 256) floats
-    if (sizeof(float) * 2 * (2 * g.n_components - 1) * static_cast<size_t>(round_up(d.d, 256)) > 227u * 1024u)
+    // the forms' coefficients stay in shared memory: 2 (2C - 1) round_up(d, 256) floats + padding
+    if (sizeof(float) * 2 * (2 * g.n_components - 1) * static_cast<size_t>(round_up(d.d, 256) / 8 * 9) > 227u * 1024u)
       return SMOES_ERR_UNSUPPORTED;
     if (!aligned16(g.X)) return SMOES_ERR_ALIGNMENT;
     if (d.T == 0) return SMOES_OK;

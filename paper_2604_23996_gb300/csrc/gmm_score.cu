@@ -55,17 +55,22 @@ __global__ void __launch_bounds__(256) k_gmm_coef(const GmmParams p) {
   }
 }
 
+// Coefficients in shared memory with one padding float after every 8 features, so that the lanes
+// of a warp, each reading its own 8 consecutive features, hit distinct banks.
+__device__ __forceinline__ int cpad(int c) { return c + (c >> 3); }
+
 template <bool kBf16>
 __global__ void __launch_bounds__(256) k_gmm_score(const GmmParams p) {
   extern __shared__ float gsm[];
   const int dpad = round_up(p.d, 256);
+  const int dps = cpad(dpad);                      // padded length of one coefficient vector
   const int F = p.F, C = p.C;
   pdl_wait();                                     // the coefficients of the kernel just before
   pdl_trigger();
   for (int f = 0; f < F; ++f)
     for (int i = threadIdx.x; i < dpad; i += 256) {
-      gsm[(2 * f) * dpad + i] = p.coef[static_cast<size_t>(f) * 2 * p.dcoef + i];
-      gsm[(2 * f + 1) * dpad + i] = p.coef[static_cast<size_t>(f) * 2 * p.dcoef + p.dcoef + i];
+      gsm[(2 * f) * dps + cpad(i)] = p.coef[static_cast<size_t>(f) * 2 * p.dcoef + i];
+      gsm[(2 * f + 1) * dps + cpad(i)] = p.coef[static_cast<size_t>(f) * 2 * p.dcoef + p.dcoef + i];
     }
   float K[kGmmMaxForms];
   bool bad = false;
@@ -85,36 +90,46 @@ __global__ void __launch_bounds__(256) k_gmm_score(const GmmParams p) {
   if (bad && blockIdx.x == 0 && threadIdx.x == 0) atomicOr(p.status, kStatusData);
   __syncthreads();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int per = kBf16 ? 8 : 4;                  // features per 16-byte load
+  constexpr int per = kBf16 ? 8 : 4;              // features per 16-byte load
+  constexpr int kIn = 8;                          // 16-byte loads of a row in flight per lane
   for (int j = blockIdx.x * 8 + warp; j < p.T; j += gridDim.x * 8) {
     float acc[kGmmMaxForms];
 #pragma unroll
     for (int f = 0; f < kGmmMaxForms; ++f) acc[f] = 0.f;
-    for (int c0 = lane * per; c0 < p.d; c0 += 32 * per) {
-      float x[8];
-      if (kBf16) {
-        const uint4 u = __ldg(reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(p.X) +
-                                                             static_cast<size_t>(j) * p.d + c0));
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    for (int cb = 0; cb < p.d; cb += 32 * per * kIn) {
+      uint4 raw[kIn];
 #pragma unroll
-        for (int r = 0; r < 4; ++r) {
-          x[2 * r] = __uint_as_float(w[r] << 16);
-          x[2 * r + 1] = __uint_as_float(w[r] & 0xffff0000u);
-        }
-      } else {
-        const float4 u = __ldg(reinterpret_cast<const float4*>(static_cast<const float*>(p.X) +
-                                                               static_cast<size_t>(j) * p.d + c0));
-        x[0] = u.x; x[1] = u.y; x[2] = u.z; x[3] = u.w;
-        x[4] = x[5] = x[6] = x[7] = 0.f;
+      for (int u = 0; u < kIn; ++u) {
+        const int c0 = cb + u * 32 * per + lane * per;
+        raw[u] = c0 < p.d ? __ldg(reinterpret_cast<const uint4*>(static_cast<const char*>(p.X) +
+                                                                 (static_cast<size_t>(j) * p.d + c0) * (kBf16 ? 2 : 4)))
+                          : make_uint4(0u, 0u, 0u, 0u);
       }
 #pragma unroll
-      for (int f = 0; f < kGmmMaxForms; ++f) {
-        if (f < F) {
-          const float* ga = gsm + (2 * f) * dpad + c0;
-          const float* gb = gsm + (2 * f + 1) * dpad + c0;
+      for (int u = 0; u < kIn; ++u) {
+        const int c0 = cb + u * 32 * per + lane * per;
+        if (c0 >= p.d) break;
+        float x[8];
+        const uint32_t w[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
+        if (kBf16) {
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            if (q < per) acc[f] = fmaf(x[q], fmaf(ga[q], x[q], gb[q]), acc[f]);
+          for (int r = 0; r < 4; ++r) {
+            x[2 * r] = __uint_as_float(w[r] << 16);
+            x[2 * r + 1] = __uint_as_float(w[r] & 0xffff0000u);
+          }
+        } else {
+#pragma unroll
+          for (int r = 0; r < 4; ++r) x[r] = __uint_as_float(w[r]);
+        }
+        const int cp = cpad(c0);
+#pragma unroll
+        for (int f = 0; f < kGmmMaxForms; ++f) {
+          if (f < F) {
+            const float* ga = gsm + (2 * f) * dps + cp;
+            const float* gb = gsm + (2 * f + 1) * dps + cp;
+#pragma unroll
+            for (int q = 0; q < per; ++q) acc[f] = fmaf(x[q], fmaf(ga[q], x[q], gb[q]), acc[f]);
+          }
         }
       }
     }
@@ -149,7 +164,7 @@ cudaError_t launch_gmm_score(const GmmParams& p, smoes_dtype dt, int n_sms, cuda
   cudaError_t e = launch_pdl(k_gmm_coef, dim3(p.dcoef / 256, p.F), dim3(256), 0, s, p);
   if (e != cudaSuccess) return e;
   const int dpad = round_up(p.d, 256);
-  const size_t smem = sizeof(float) * 2 * static_cast<size_t>(p.F) * dpad;
+  const size_t smem = sizeof(float) * 2 * static_cast<size_t>(p.F) * (dpad + dpad / 8);
   if (smem > 227u * 1024u) return cudaErrorInvalidConfiguration;
   int grid = (p.T + 7) / 8;
   if (grid > 4 * n_sms) grid = 4 * n_sms;
