@@ -6,14 +6,17 @@
 //
 // A work item is (sequence, head, 128-query tile); items run longest first on persistent CTAs.
 // Per 128-key block the tensor cores form S = Q K^T into one of two TMEM buffers (tcgen05,
-// TMA-fed). Four softmax warps (one query row per thread) keep the online state: the running
-// maximum used for the exponentials, the normaliser l and the vision mass a = sum P m; P goes to
-// shared memory in bf16 (as FlashAttention passes it to the tensor cores) and the tensor cores
-// accumulate O += P V in TMEM. The maximum in use is only raised when a block's maximum exceeds it
-// by more than 2^8 (then O, l and a are rescaled once), so the exponentials stay below 2^8 and the
-// rescale is rare. At the end of an item O / l leaves through a TMA store, a / l goes to the
-// per-head partials, and the last head of each (sequence, query tile) to finish averages the heads
-// in fixed order and writes M (optionally blended with the carried score by eq. 4).
+// TMA-fed). Two softmax warp groups (four warps each, one query row per thread) take the two
+// halves of the block's keys and keep independent online states: the running maximum used for
+// the exponentials, the normaliser l and the vision mass a = sum P m. Each half writes its P (bf16,
+// as FlashAttention passes it to the tensor cores) to its half of a shared-memory tile and the
+// tensor cores accumulate O_h += P_h V_h into the half's own TMEM accumulator. The maximum in use
+// is only raised when a block's maximum exceeds it by more than 2^8 (then O_h, l and a are
+// rescaled), so the exponentials stay below 2^8 and rescales are rare. At the end of an item the
+// first group merges the halves (O = (2^(m0-m) O_0 + 2^(m1-m) O_1) / l), O leaves through a TMA
+// store, a / l goes to the per-head partials, and the last head of each (sequence, query tile) to
+// finish averages the heads in fixed order and writes M (optionally blended with the carried score
+// by eq. 4).
 #include <cuda_bf16.h>
 #include <math_constants.h>
 
@@ -28,11 +31,12 @@ constexpr int kFT = 128;                       // queries per tile, keys per blo
 constexpr int kFHd = 128;                      // head dimension handled here
 constexpr uint32_t kFTile = kFT * kFHd * 2;    // bytes of a Q tile, K or V block, P or O tile
 constexpr int kFStages = 2;                    // K/V blocks in flight
-constexpr int kFThreads = 64 + 128;            // producer, MMA issuer, four softmax warps
+constexpr int kFHalf = kFT / 2;                // keys of a block per softmax group
+constexpr int kFThreads = 64 + 2 * 128;        // producer, MMA issuer, two softmax groups
 constexpr float kRescale = 8.f;                // raise the maximum in use only past +2^8
 
 struct FwdAttnLayout {
-  uint32_t q, k, v, pbuf, stg, bars, total;
+  uint32_t q, k, v, pbuf, stg, mrg, bars, total;
 };
 
 // Q tile, K/V stages, the P tile (also the staging of O at the end of an item), per-stage key
@@ -45,7 +49,8 @@ __host__ __device__ inline FwdAttnLayout fwd_attn_layout() {
   L.v = o;    o += kFStages * kFTile;
   L.pbuf = o; o += kFTile;
   L.stg = o;  o += kFStages * 2u * kFT * 4u;
-  L.bars = o; o += 8u * (4u * kFStages + 16u) + 32u;
+  L.mrg = o;  o += 2u * 3u * kFT * 4u;            // second half's (max, l, a) per row, by item parity
+  L.bars = o; o += 8u * (4u * kFStages + 24u) + 32u;
   L.total = o + 1024u;
   return L;
 }
@@ -99,20 +104,22 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
   uint64_t* bars = reinterpret_cast<uint64_t*>(base + L.bars);
   uint64_t* kvfull = bars;                    // [kFStages] K, V and the key terms have landed
   uint64_t* kvempty = bars + kFStages;        // [kFStages] the block's P V has completed
+  float* mrg = reinterpret_cast<float*>(base + L.mrg);   // [item parity][max | l | a][128]
   uint64_t* q_full = bars + 2 * kFStages;
   uint64_t* q_empty = q_full + 1;             // the item's last S has read Q
   uint64_t* s_full = q_full + 2;              // [2]
-  uint64_t* s_empty = q_full + 4;             // [2] count 128
-  uint64_t* p_full = q_full + 6;              // count 128
-  uint64_t* p_empty = q_full + 7;             // the block's P V has read P
-  uint64_t* o_full = q_full + 8;              // the item's last P V has completed
-  uint64_t* o_empty = q_full + 9;             // count 128: O read by the epilogue
-  uint64_t* stg_full = q_full + 10;           // count 128: O staged
-  uint64_t* stg_free = q_full + 11;           // the O store has read the staging
-  uint64_t* out_bar = q_full + 12;            // count 128: head partials written
-  uint64_t* dec_bar = q_full + 13;            // the tile's last-head decision is known
-  uint64_t* drain = q_full + 14;              // all of the MMA warp's work has completed
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 15);
+  uint64_t* s_empty = q_full + 4;             // [2] count 256 (both groups)
+  uint64_t* p_full = q_full + 6;              // [2 halves] count 128
+  uint64_t* p_empty = q_full + 8;             // [2 halves] the half's P V has read its P
+  uint64_t* o_full = q_full + 10;             // the item's last P V has completed
+  uint64_t* o_empty = q_full + 11;            // count 128: O read by the epilogue
+  uint64_t* stg_full = q_full + 12;           // count 128: O staged
+  uint64_t* stg_free = q_full + 13;           // the O store has read the staging
+  uint64_t* out_bar = q_full + 14;            // count 128: head partials written
+  uint64_t* dec_bar = q_full + 15;            // the tile's last-head decision is known
+  uint64_t* drain = q_full + 16;              // all of the MMA warp's work has completed
+  uint64_t* mrg_bar = q_full + 17;            // [2] count 128: the second half's state is handed over
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 19);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
   uint32_t* decision = reinterpret_cast<uint32_t*>(tmem_slot + 2);
 
@@ -129,10 +136,11 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
     mbar_init(q_empty, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(s_full + i, 1);
-      mbar_init(s_empty + i, 128);
+      mbar_init(s_empty + i, 256);
+      mbar_init(p_full + i, 128);
+      mbar_init(p_empty + i, 1);
+      mbar_init(mrg_bar + i, 128);
     }
-    mbar_init(p_full, 128);
-    mbar_init(p_empty, 1);
     mbar_init(o_full, 1);
     mbar_init(o_empty, 128);
     mbar_init(stg_full, 128);
@@ -150,7 +158,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *tmem_slot;             // S buffers at columns 0 and 128, O at 256
+  const uint32_t tmem = *tmem_slot;             // S buffers at columns 0 and 128, O_0 at 256, O_1 at 384
   pdl_wait();                                   // Q, K, V, the scores and M of earlier work
   pdl_trigger();
   const int n_items = p.n_items;
@@ -236,20 +244,23 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
             if (j == nb - 1) umma_commit(q_empty);
           }
           if (j > 0) {
-            // O += P_{j-1} V_{j-1} once the softmax has written P_{j-1}
+            // O_h += P_h V_h of block j - 1, each half once its softmax group has written its P
             const long gp = g - 1;                              // global index of block j - 1
-            if (!mbar_wait(p_full, static_cast<uint32_t>(gp) & 1u, wc)) { ok = false; break; }
-            if (j == 1 && !mbar_wait(o_empty, (static_cast<uint32_t>(n) & 1u) ^ 1u, wc)) { ok = false; break; }
-            tc_fence_after();
             const uint32_t pa = smem_u32(pb);
             const uint32_t vb = smem_u32(vs + pst * kFTile);
+            for (int hf = 0; hf < 2 && ok; ++hf) {
+              if (!mbar_wait(p_full + hf, static_cast<uint32_t>(gp) & 1u, wc)) { ok = false; break; }
+              if (j == 1 && hf == 0 && !mbar_wait(o_empty, (static_cast<uint32_t>(n) & 1u) ^ 1u, wc)) { ok = false; break; }
+              tc_fence_after();
 #pragma unroll
-            for (int kk = 0; kk < kFT / 16; ++kk) {      // K = 16 keys per step
-              const uint64_t da = sdesc_sw128(pa + (kk >> 2) * (kFTile / 2) + (kk & 3) * 32, 16, 1024);
-              const uint64_t dv = sdesc_sw128(vb + kk * 2048, kFTile / 2, 1024);
-              umma_bf16(tm_o, da, dv, id_o, (j > 1 || kk > 0) ? 1u : 0u);
+              for (int kk = 0; kk < kFHalf / 16; ++kk) {   // K = 16 keys per step
+                const uint64_t da = sdesc_sw128(pa + hf * (kFTile / 2) + kk * 32, 16, 1024);
+                const uint64_t dv = sdesc_sw128(vb + (hf * (kFHalf / 16) + kk) * 2048, kFTile / 2, 1024);
+                umma_bf16(tm_o + static_cast<uint32_t>(hf * kFHd), da, dv, id_o, (j > 1 || kk > 0) ? 1u : 0u);
+              }
+              umma_commit(p_empty + hf);
             }
-            umma_commit(p_empty);
+            if (!ok) break;
             umma_commit(kvempty + pst);
             if (++pst == kFStages) pst = 0;
             if (j == nb) umma_commit(o_full);
@@ -267,11 +278,13 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
       mbar_wait(drain, 0, wd);
     }
   } else {
-    // -------------------------------------------------------------- softmax warps (4) + epilogue
+    // -------------------------------------------------------------- softmax groups (2 x 4 warps)
+    const int hf = (warp - 2) >> 2;              // half of each block's keys
     const int lg = warp & 3;                     // TMEM lane quarter of this warp
     const int row = lg * 32 + lane;              // query row of the tile
-    const int gtid = threadIdx.x - 64;
+    const int gtid = (threadIdx.x - 64) & 127;   // thread of the group
     const uint32_t lane_off = static_cast<uint32_t>(lg * 32) << 16;
+    const uint32_t to = tmem + lane_off + 256u + static_cast<uint32_t>(hf * kFHd);   // O_hf
     bool ok = true;
     long g = 0;
     int st = 0;
@@ -290,29 +303,40 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
         const float* kts = kt + st * 2 * kFT;
         const uint8_t* mkb = reinterpret_cast<const uint8_t*>(kts + kFT);
         const bool diag = p.causal && j == it.qt;
-        const uint32_t ts = tmem + lane_off + static_cast<uint32_t>(sb * kFT);
-        auto logit2 = [&](float v, int key) {     // log2-scaled logit of this row and key
-          const float b = p.key_bias ? kts[key] * 1.4426950408889634f : 0.f;
-          const float t = fmaf(v, p.scale_log2, b);
-          return (diag && key > row) ? -CUDART_INF_F : t;
-        };
-        // pass 1: the block's row maximum
-        float mx = -CUDART_INF_F;
-#pragma unroll 1
-        for (int c = 0; c < kFT / 32; ++c) {
+        const uint32_t ts = tmem + lane_off + static_cast<uint32_t>(sb * kFT + hf * kFHalf);
+        // the half's 64 logits of this row, log2-scaled, masked above the diagonal
+        float t[kFHalf];
+        {
           float v[32];
-          tmem_ld32(ts + 32u * c, v);
+          tmem_ld32(ts, v);
 #pragma unroll
-          for (int q = 0; q < 32; ++q) mx = fmaxf(mx, logit2(v[q], c * 32 + q));
+          for (int q = 0; q < 32; ++q) t[q] = v[q];
+          tmem_ld32(ts + 32u, v);
+#pragma unroll
+          for (int q = 0; q < 32; ++q) t[32 + q] = v[q];
+        }
+        tc_fence_before();
+        mbar_arrive(s_empty + sb);               // the S buffer may be rewritten
+        float mx = -CUDART_INF_F;
+#pragma unroll
+        for (int q = 0; q < kFHalf; ++q) {
+          const int key = hf * kFHalf + q;
+          const float b = p.key_bias ? kts[key] * 1.4426950408889634f : 0.f;
+          t[q] = (diag && key > row) ? -CUDART_INF_F : fmaf(t[q], p.scale_log2, b);
+          mx = fmaxf(mx, t[q]);
         }
         const float m_new = fmaxf(m_used, mx);
         const bool raise = j == 0 || m_new > m_used + kRescale;
-        // P of the previous block has been read by its P V (and O updated) before P or O change
-        if (j > 0 && !mbar_wait(p_empty, static_cast<uint32_t>(g - 1) & 1u, wc)) { ok = false; break; }
-        if (__any_sync(0xffffffffu, raise && j > 0)) {          // rescale O, l and a (rare)
+        // the half's previous P V has read its P and updated O_hf before either changes; at the
+        // first block of an item the staging of the previous item's O must have been stored
+        if (j > 0) {
+          if (!mbar_wait(p_empty + hf, static_cast<uint32_t>(g - 1) & 1u, wc)) { ok = false; break; }
+        } else if (n > 0) {
+          if (!mbar_wait(stg_free, static_cast<uint32_t>(n - 1) & 1u, wc)) { ok = false; break; }
+        }
+        if (__any_sync(0xffffffffu, raise && j > 0)) {          // rescale O_hf, l and a (rare)
           tc_fence_after();
-          const float alpha = (raise && j > 0) ? ex2f(m_used - m_new) : 1.f;
-          const uint32_t to = tmem + lane_off + 256u;
+          const float alpha = (raise && j > 0) ? (m_used == -CUDART_INF_F ? 0.f : ex2f(m_used - m_new)) : 1.f;
 #pragma unroll 1
           for (int c = 0; c < kFHd / 32; ++c) {
             float v[32];
@@ -325,47 +349,61 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
           a *= alpha;
         }
         if (raise) m_used = m_new;
-        // pass 2: P = 2^(logit - max in use) in bf16 to shared memory; l and the vision mass
-#pragma unroll 1
-        for (int c = 0; c < kFT / 32; ++c) {
-          float v[32];
-          tmem_ld32(ts + 32u * c, v);
-          uint32_t pk[16];
+        // P = 2^(logit - max in use) in bf16 to the half's atom of the P tile; l and the mass. A
+        // half whose keys are all above the diagonal so far (max -inf) has P = 0.
+        const float msub = m_used == -CUDART_INF_F ? 0.f : m_used;
+        uint32_t pk[kFHalf / 2];
 #pragma unroll
-          for (int q = 0; q < 32; q += 2) {
-            const int k0 = c * 32 + q;
-            const float p0 = ex2f(logit2(v[q], k0) - m_used), p1 = ex2f(logit2(v[q + 1], k0 + 1) - m_used);
-            const float m0 = kFloatM ? kts[kFT + k0] : (mkb[k0] ? 1.f : 0.f);
-            const float m1 = kFloatM ? kts[kFT + k0 + 1] : (mkb[k0 + 1] ? 1.f : 0.f);
-            l += p0 + p1;
-            a = fmaf(p0, m0, fmaf(p1, m1, a));
-            pk[q >> 1] = pack2_bf16(p0, p1);
-          }
-          uint8_t* prow = pb + (c >> 1) * (kFTile / 2) + row * 128;
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const uint32_t chunk = static_cast<uint32_t>((c & 1) * 4 + u) ^ static_cast<uint32_t>(row & 7);
-            *reinterpret_cast<uint4*>(prow + (chunk << 4)) = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
-          }
+        for (int q = 0; q < kFHalf; q += 2) {
+          const int k0 = hf * kFHalf + q;
+          const float p0 = ex2f(t[q] - msub), p1 = ex2f(t[q + 1] - msub);
+          const float m0 = kFloatM ? kts[kFT + k0] : (mkb[k0] ? 1.f : 0.f);
+          const float m1 = kFloatM ? kts[kFT + k0 + 1] : (mkb[k0 + 1] ? 1.f : 0.f);
+          l += p0 + p1;
+          a = fmaf(p0, m0, fmaf(p1, m1, a));
+          pk[q >> 1] = pack2_bf16(p0, p1);
         }
-        tc_fence_before();
-        mbar_arrive(s_empty + sb);
+        uint8_t* prow = pb + hf * (kFTile / 2) + row * 128;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const uint32_t chunk = static_cast<uint32_t>(u) ^ static_cast<uint32_t>(row & 7);
+          *reinterpret_cast<uint4*>(prow + (chunk << 4)) = make_uint4(pk[4 * u], pk[4 * u + 1], pk[4 * u + 2], pk[4 * u + 3]);
+        }
         fence_proxy_async_smem();
-        mbar_arrive(p_full);
+        mbar_arrive(p_full + hf);
         if (++st == kFStages) { st = 0; ph ^= 1u; }
       }
       if (!ok) break;
-      // epilogue: O / l through the staging (the P buffer, free once the last P V completed)
+      float* mb = mrg + (n & 1) * 3 * kFT;
+      if (hf == 1) {                             // hand the half's state to the first group
+        mb[row] = m_used;
+        mb[kFT + row] = l;
+        mb[2 * kFT + row] = a;
+        mbar_arrive(mrg_bar + (n & 1));
+        continue;
+      }
+      // epilogue (first group): merge the halves, O / l through the staging (the P tile, free
+      // once the last P V completed)
       if (!mbar_wait(o_full, static_cast<uint32_t>(n) & 1u, wc)) { ok = false; break; }
+      if (!mbar_wait(mrg_bar + (n & 1), static_cast<uint32_t>(n >> 1) & 1u, wc)) { ok = false; break; }
       tc_fence_after();
+      const float m1 = mb[row], l1 = mb[kFT + row], a1 = mb[2 * kFT + row];
+      const float mm = fmaxf(m_used, m1);                   // finite: the first half sees key 0
+      const float c0 = ex2f(m_used - mm), c1 = m1 == -CUDART_INF_F ? 0.f : ex2f(m1 - mm);
+      l = l * c0 + l1 * c1;
+      a = a * c0 + a1 * c1;
       const float il = 1.f / l;
+      const float s0 = c0 * il, s1 = c1 * il;
+      const uint32_t o0 = tmem + lane_off + 256u;
 #pragma unroll 1
       for (int c = 0; c < kFHd / 32; ++c) {
-        float v[32];
-        tmem_ld32(tmem + lane_off + 256u + 32u * c, v);
+        float v[32], w[32];
+        tmem_ld32(o0 + 32u * c, v);
+        tmem_ld32(o0 + kFHd + 32u * c, w);
         uint32_t pk[16];
 #pragma unroll
-        for (int q = 0; q < 32; q += 2) pk[q >> 1] = pack2_bf16(v[q] * il, v[q + 1] * il);
+        for (int q = 0; q < 32; q += 2)
+          pk[q >> 1] = pack2_bf16(fmaf(v[q], s0, w[q] * s1), fmaf(v[q + 1], s0, w[q + 1] * s1));
         uint8_t* orow = pb + (c >> 1) * (kFTile / 2) + row * 128;
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
@@ -417,7 +455,7 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
         reinterpret_cast<float2*>(p.M)[tok] = make_float2(mv, 1.f - mv);
       }
     }
-    if (gtid == 0) tma_store_wait_all<0>();
+    if (hf == 0 && gtid == 0) tma_store_wait_all<0>();
   }
 
   tc_fence_before();
