@@ -458,6 +458,9 @@ k_attn_fwd(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUte
     if (hf == 0 && gtid == 0) tma_store_wait_all<0>();
   }
 
+  // the role branches leave single lanes running on their own: the warp reconverges before
+  // the block barrier, so that no thread passes it while another of its warp is still working
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();

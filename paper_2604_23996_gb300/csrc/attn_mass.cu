@@ -415,6 +415,9 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     }
   }
 
+  // the role branches leave single lanes running on their own: the warp reconverges before
+  // the block barrier, so that no thread passes it while another of its warp is still working
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();

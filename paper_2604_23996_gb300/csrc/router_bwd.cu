@@ -587,6 +587,9 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     }
   }
 
+  // the role branches leave single lanes running on their own: the warp reconverges before
+  // the block barrier, so that no thread passes it while another of its warp is still working
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();

@@ -118,21 +118,22 @@ __device__ __noinline__ void sample_reduce(const FwdParams& p, int s, float* red
     pe = p.ws.sample_pieces[s + 1];
     nt = p.ws.offsets[s + 1] - p.ws.offsets[s];
   }
-  // lane l sums value 32c + l over the sample's pieces in piece order, 16 loads in flight
+  // lane l sums value 32c + l over the sample's pieces in piece order, 32 loads in flight (one
+  // round of memory latency per 32 pieces: the reduction sits on the forward's tail)
 #pragma unroll 1
   for (int c = 0; c * 32 < NV; ++c) {
     const int v = 32 * c + lane;
     const bool in = v < NV;
     float acc = 0.f;
 #pragma unroll 1
-    for (int q0 = pb; q0 < pe; q0 += 16) {
+    for (int q0 = pb; q0 < pe; q0 += 32) {
       const float* src = p.ws.pieces + static_cast<size_t>(q0) * dm.pstride + (in ? v : 0);
-      float t[16];
+      float t[32];
 #pragma unroll
-      for (int i = 0; i < 16; ++i)
+      for (int i = 0; i < 32; ++i)
         t[i] = (in && !dry && q0 + i < pe) ? __ldcg(src + static_cast<size_t>(i) * dm.pstride) : 0.f;
 #pragma unroll
-      for (int i = 0; i < 16; ++i) acc += t[i];
+      for (int i = 0; i < 32; ++i) acc += t[i];
     }
     if (in) red[v] = acc;
   }
@@ -1176,6 +1177,9 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     if (!kGauss && warp < 2) perm_tail<KM>(p, t_beg, t_end, threadIdx.x, 2, 1, ctot, ps, perm_go, wc);
   }
 
+  // the role branches leave single lanes running on their own: the warp reconverges before
+  // the block barrier, so that no thread passes it while another of its warp is still working
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -1318,15 +1322,39 @@ k_router_fwd_f32(const FwdParams p) {
   __threadfence();
   if (t == 0) p.tile_ticket[tile] = 0u;                  // ready for the next call
   const float* pt = p.f32_part + static_cast<size_t>(tile * nck) * (E + 1) * 128;
-  for (int i = 0; i < (E16 + 1) / 2 + 1; ++i) {
-    const int e = 2 * i + h;
-    if (e > E16) break;
-    float z = 0.f;
-    if (e < E || (kGauss && e == E)) {
-      for (int c = 0; c < nck; ++c) z += __ldcg(pt + static_cast<size_t>(c) * (E + 1) * 128 + e * 128 + r);
+  // thread (r, h) sums values e = 2i + h (the logits, then the log-likelihood difference at e = E)
+  // over the chunks in chunk order; the loads of CB chunks of every e are issued together
+  {
+    constexpr int NI = EB / 2 + 1;
+    constexpr int CB = EB <= 16 ? 4 : EB <= 32 ? 2 : 1;
+    float zz[NI];
+#pragma unroll
+    for (int i = 0; i < NI; ++i) zz[i] = 0.f;
+#pragma unroll 1
+    for (int c0 = 0; c0 < nck; c0 += CB) {
+      float t[NI][CB];
+#pragma unroll
+      for (int i = 0; i < NI; ++i) {
+        const int e = 2 * i + h;
+        const bool on = e < E || (kGauss && e == E);
+#pragma unroll
+        for (int u = 0; u < CB; ++u)
+          t[i][u] = (on && c0 + u < nck)
+                        ? __ldcg(pt + static_cast<size_t>(c0 + u) * (E + 1) * 128 + e * 128 + r) : 0.f;
+      }
+#pragma unroll
+      for (int i = 0; i < NI; ++i) {
+#pragma unroll
+        for (int u = 0; u < CB; ++u)
+          if (c0 + u < nck) zz[i] += t[i][u];
+      }
     }
-    if (e < E16) zs[r * (E16 + 1) + e] = z;            // padding experts: logit 0, masked below
-    if (kGauss && e == E) dll_s[r] = z;
+#pragma unroll
+    for (int i = 0; i < NI; ++i) {
+      const int e = 2 * i + h;
+      if (e < E16) zs[r * (E16 + 1) + e] = zz[i];       // padding experts: logit 0, masked below
+      if (kGauss && e == E) dll_s[r] = zz[i];
+    }
   }
   __syncthreads();
   {
