@@ -403,18 +403,21 @@ class Step:
                              is_vision=torch.from_numpy(aw.is_vision).to(dev))
         self.parts = (([("attn", self.score)] if self.use_attn else [])
                       + [("fwd+permute", self.fwd_perm), ("bwd", self.bwd)])
-        # our kernels per step: attention 1; fwd + permutation 1 (one cooperative launch; fp32:
-        # Gaussian coefficients 1, forward 1, permutation 1); bwd 3 (dz prep, main, dW reduce;
-        # fp32: main, dW reduce)
-        fwd_launches = ((0 if self.use_attn else 1) + 2) if self.f32 else 1
-        self.launches = (1 if self.use_attn else 0) + fwd_launches + (2 if self.f32 else 3)
+        # our kernels per step, as the library reports them for this plan: the attention score,
+        # the forward with the permutation (one launch when the permutation is fused into the
+        # forward kernel, else two), the backward (dz prep, main, dW sum; fp32: main, dW sum)
+        plan = self.r.plan
+        self.fwd_launches = bd.smoes_call_launches(plan, bd.SMOES_CALL_ROUTER_FWD_PERMUTE)
+        self.launches = ((bd.smoes_call_launches(plan, bd.SMOES_CALL_ATTN_SCORE) if self.use_attn else 0)
+                         + self.fwd_launches + bd.smoes_call_launches(plan, bd.SMOES_CALL_ROUTER_BWD))
+        assert min(self.fwd_launches, self.launches) > 0
 
     def score(self, X=None, Q=None, K=None):
         a = self.attn if Q is None else dict(self.attn, Q=Q, K=K)
         self.r.modality_score(self.bd.SMOES_SCORE_ATTN, self.Ma, attn=a)
 
     def fwd_perm(self, X=None, W=None, mu=None, var=None):
-        # the forward and the bin permutation of its top-k: one launch on the bf16 path
+        # the forward and the bin permutation of its top-k
         X = self.X if X is None else X
         W = self.W if W is None else W
         if self.use_attn:
@@ -806,7 +809,9 @@ def main():
             call = "fwd" if name.startswith("fwd") else "bwd"
             by = fwd_bytes if call == "fwd" else bwd_bytes
             ach = by / (ms * 1e-3) / 1e9
-            kern = ("smoes_router_fwd_permute (k_router_fwd_tc, one launch)" if call == "fwd" and not st.f32
+            fwd_kern = ("smoes_router_fwd_permute (k_router_fwd_tc, one launch)" if st.fwd_launches == 1
+                        else "smoes_router_fwd_permute (k_router_fwd_tc + k_perm)")
+            kern = (fwd_kern if call == "fwd" and not st.f32
                     else "smoes_router_bwd (k_dz_prep + k_router_bwd_tc + k_dw_reduce)" if not st.f32
                     else f"smoes_router_{call} (fp32 path)")
             tkey = args.config if args.tokens is None else f"{args.config}_T{wl.T}"

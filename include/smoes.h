@@ -56,6 +56,14 @@ typedef enum {
 
 typedef enum { SMOES_GATE_SOFTMAX = 0, SMOES_GATE_SIGMOID = 1 } smoes_gate;
 
+typedef enum {
+  SMOES_CALL_ROUTER_FWD = 0,          /* smoes_router_fwd                                 */
+  SMOES_CALL_ROUTER_FWD_PERMUTE = 1,  /* smoes_router_fwd_permute                         */
+  SMOES_CALL_ROUTER_BWD = 2,          /* smoes_router_bwd                                 */
+  SMOES_CALL_BIN_PERMUTE = 3,         /* smoes_bin_permute                                */
+  SMOES_CALL_ATTN_SCORE = 4           /* smoes_modality_score with SMOES_SCORE_ATTN       */
+} smoes_call;
+
 typedef struct smoes_plan_s* smoes_plan;
 
 /* Shape and routing metadata of one router layer (Secs. 3.1, 3.3).
@@ -158,6 +166,13 @@ size_t smoes_workspace_bytes(smoes_plan plan);
  * Call once after allocating the workspace (and again after any device-side error), on the
  * stream that later calls use. */
 smoes_status smoes_workspace_init(smoes_plan plan, void* ws, size_t ws_bytes, cudaStream_t stream);
+
+/* Kernel launches one call makes on this plan (a host query: no GPU work, no allocation). Nothing
+ * else is enqueued besides these kernels, except a cudaMemsetAsync of the outputs of empty
+ * (T == 0) calls, counted as 0. smoes_router_fwd_permute is one launch when the permutation
+ * runs inside the forward kernel (SMOES_BF16 plans of at most two 128-token tiles per SM), two
+ * otherwise. Returns -1 for a null plan or an unknown call. */
+int smoes_call_launches(smoes_plan plan, smoes_call call);
 
 const char* smoes_status_string(smoes_status status);
 

@@ -26,6 +26,8 @@ STATUS_NAMES = {0: "SMOES_OK", -1: "SMOES_ERR_INVALID_ARG", -2: "SMOES_ERR_UNSUP
 SMOES_F32, SMOES_BF16 = 0, 1
 SMOES_GATE_SOFTMAX, SMOES_GATE_SIGMOID = 0, 1
 SMOES_SCORE_PROVIDED, SMOES_SCORE_GAUSS, SMOES_SCORE_ATTN, SMOES_SCORE_GMM = 0, 1, 2, 3
+(SMOES_CALL_ROUTER_FWD, SMOES_CALL_ROUTER_FWD_PERMUTE, SMOES_CALL_ROUTER_BWD, SMOES_CALL_BIN_PERMUTE,
+ SMOES_CALL_ATTN_SCORE) = 0, 1, 2, 3, 4
 
 
 class SmoesError(RuntimeError):
@@ -71,6 +73,7 @@ _sig = {
     "smoes_workspace_init": (_i, [_vp, _vp, _sz, _vp]),
     "smoes_status_string": (C.c_char_p, [_i]),
     "smoes_plan_set_wait_limit": (_i, [_vp, C.c_uint64]),
+    "smoes_call_launches": (_i, [_vp, _i]),
     "smoes_read_device_status": (_i, [_vp, _vp, _vp, C.POINTER(C.c_int32)]),
     "smoes_modality_score": (_i, [_vp, _i, C.POINTER(ScoreArgs), _vp, _vp, _sz, _vp]),
     "smoes_router_fwd": (_i, [_vp, _vp, _vp, _vp, C.POINTER(GaussArgs), _vp, _vp, _vp, _vp, _vp,
@@ -132,6 +135,11 @@ def smoes_plan_create(T, d, E, k, n_bins, sample_offsets, expert_bin, dtype, ren
 
 def smoes_plan_set_wait_limit(plan, limit_ns: int) -> int:
     return _lib.smoes_plan_set_wait_limit(plan, int(limit_ns))
+
+
+def smoes_call_launches(plan, call: int) -> int:
+    """Kernel launches one call makes on this plan (host query)."""
+    return _lib.smoes_call_launches(plan, int(call))
 
 
 def smoes_plan_destroy(plan):

@@ -170,6 +170,16 @@ smoes_status check_ws(const smoes_plan_s* P, const void* ws, size_t ws_bytes) {
 
 smoes_status cuda_status(cudaError_t e) { return e == cudaSuccess ? SMOES_OK : SMOES_ERR_CUDA; }
 
+// The permutation runs inside the forward launch on the tensor-core path when every CTA holds at
+// most two tiles (the fused scatter runs after a CTA's last tile, serially over its tokens: with
+// many tiles per CTA the standalone permutation, spread over the whole GPU, is faster).
+bool fuse_permute(const smoes_plan_s* P) {
+  const smoes_router_desc& d = P->desc;
+  const int fwd_tiles = (d.T + kFwdBM - 1) / kFwdBM;
+  return d.dtype == SMOES_BF16 && d.T > 0 && d.n_bins <= kMaxBins && d.E <= kMaxExperts &&
+         fwd_tiles <= 2 * P->n_sms;
+}
+
 // The forward of smoes_router_fwd; perm: the fused permutation's outputs (tensor-core path), or null.
 smoes_status router_fwd(smoes_plan P, const void* X, const void* W, const float* M_in,
                         const smoes_gauss_args* gauss, float* M_out, int32_t* topk_idx,
@@ -419,6 +429,20 @@ smoes_status smoes_workspace_init(smoes_plan P, void* ws, size_t ws_bytes, cudaS
   return cuda_status(e);
 }
 
+int smoes_call_launches(smoes_plan P, smoes_call call) {
+  if (!P) return -1;
+  const smoes_router_desc& d = P->desc;
+  const int any = d.T > 0 ? 1 : 0;
+  switch (call) {
+    case SMOES_CALL_ROUTER_FWD: return any;
+    case SMOES_CALL_ROUTER_FWD_PERMUTE: return any ? (fuse_permute(P) ? 1 : 2) : 0;
+    case SMOES_CALL_ROUTER_BWD: return any ? (d.dtype == SMOES_BF16 ? 3 : 2) : 0;  // (dz prep,) main, dW sum
+    case SMOES_CALL_BIN_PERMUTE: return any;
+    case SMOES_CALL_ATTN_SCORE: return any;
+  }
+  return -1;
+}
+
 smoes_status smoes_read_device_status(smoes_plan P, const void* ws, cudaStream_t stream,
                                       int32_t* n_absent) {
   if (!P || !ws) return SMOES_ERR_INVALID_ARG;
@@ -603,13 +627,8 @@ smoes_status smoes_router_fwd_permute(smoes_plan P, const void* X, const void* W
   if (!bin_offsets || !dispatch) return SMOES_ERR_INVALID_ARG;
   if (expert_counts && !is_vision) return SMOES_ERR_INVALID_ARG;
   if (d.T > 0 && (!perm_token || !perm_mask)) return SMOES_ERR_INVALID_ARG;
-  // inside the forward launch on the tensor-core path when every CTA holds at most two tiles
-  // (the fused scatter runs after a CTA's last tile, serially over its tokens: with many tiles
-  // per CTA the standalone permutation, spread over the whole GPU, is faster); otherwise the two
-  // calls in order
-  const int fwd_tiles = (d.T + kFwdBM - 1) / kFwdBM;
-  if (d.dtype == SMOES_BF16 && d.T > 0 && d.n_bins <= kMaxBins && d.E <= kMaxExperts &&
-      fwd_tiles <= 2 * P->n_sms) {
+  // inside the forward launch when fuse_permute(P); otherwise the two calls in order
+  if (fuse_permute(P)) {
     FusedPerm f{};
     f.home = home;
     f.is_vision = is_vision;

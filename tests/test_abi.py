@@ -92,6 +92,32 @@ def test_wait_limit_setter(bd):
     bd.smoes_plan_destroy(plan)
 
 
+def test_call_launch_counts(bd):
+    # the host's SM count decides the fused permutation: 2 tiles per SM at most (any GPU has more
+    # than 8 SMs and fewer than 4096)
+    code, small = _plan(bd)                                                 # 1 tile
+    assert code == 0
+    assert bd.smoes_call_launches(small, bd.SMOES_CALL_ROUTER_FWD) == 1
+    assert bd.smoes_call_launches(small, bd.SMOES_CALL_ROUTER_FWD_PERMUTE) == 1
+    assert bd.smoes_call_launches(small, bd.SMOES_CALL_ROUTER_BWD) == 3    # dz prep, main, dW sum
+    assert bd.smoes_call_launches(small, bd.SMOES_CALL_BIN_PERMUTE) == 1
+    assert bd.smoes_call_launches(small, bd.SMOES_CALL_ATTN_SCORE) == 1
+    assert bd.smoes_call_launches(small, 99) == -1
+    assert bd.smoes_call_launches(None, bd.SMOES_CALL_ROUTER_FWD) == -1
+    code, big = _plan(bd, T=1 << 20, sample_offsets=[0, 1 << 20])           # 8192 tiles
+    assert code == 0
+    assert bd.smoes_call_launches(big, bd.SMOES_CALL_ROUTER_FWD_PERMUTE) == 2
+    code, f32 = _plan(bd, dtype=bd.SMOES_F32)
+    assert code == 0
+    assert bd.smoes_call_launches(f32, bd.SMOES_CALL_ROUTER_FWD_PERMUTE) == 2
+    assert bd.smoes_call_launches(f32, bd.SMOES_CALL_ROUTER_BWD) == 2      # main, dW sum
+    code, empty = bd.smoes_plan_create(0, 64, 16, 2, 4, [0], np.arange(16) // 4, bd.SMOES_BF16)
+    assert code == 0
+    assert bd.smoes_call_launches(empty, bd.SMOES_CALL_ROUTER_BWD) == 0
+    for p in (small, big, f32, empty):
+        bd.smoes_plan_destroy(p)
+
+
 def test_empty_batch_plan(bd):
     code, plan = bd.smoes_plan_create(0, 64, 16, 2, 4, [0], np.arange(16) // 4, bd.SMOES_BF16)
     assert code == 0
