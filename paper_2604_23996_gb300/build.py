@@ -17,8 +17,9 @@ LIBDIR = os.path.join(PKG, "lib")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(LIBDIR, "libsmoes.so")
 
-SOURCES = ["api.cu", "router_fwd.cu", "router_bwd.cu", "bin_permute.cu", "gauss_score.cu", "gmm_score.cu",
-           "gauss_stats.cu", "bin_balance.cu", "attn_mass.cu", "attn_fwd.cu"]
+SOURCES = ["api.cu", "router_fwd.cu", "router_fwd_var.cu", "router_bwd.cu", "bin_permute.cu",
+           "gauss_score.cu", "gmm_score.cu", "gauss_stats.cu", "bin_balance.cu", "attn_mass.cu",
+           "attn_fwd.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I" + INCLUDE, "-I" + CSRC]
 

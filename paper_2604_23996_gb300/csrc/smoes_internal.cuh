@@ -289,6 +289,9 @@ cudaError_t launch_pdl(void (*k)(KArgs...), dim3 grid, dim3 block, size_t smem, 
 cudaError_t launch_router_fwd_bf16(const FwdParams& p, const CUtensorMap& tmX,
                                    const CUtensorMap& tmW, const CUtensorMap* tmG, int n_sms,
                                    cudaStream_t s);
+cudaError_t launch_router_fwd_bf16_var(const FwdParams& p, const CUtensorMap& tmX,
+                                       const CUtensorMap& tmW, const CUtensorMap* tmG, int n_sms,
+                                       cudaStream_t s);   // router variants compiled in
 cudaError_t launch_router_fwd_f32(const FwdParams& p, cudaStream_t s);
 int f32_chunks(int d);     // feature chunks of the fp32 forward and backward (128 features each)
 cudaError_t launch_router_bwd_bf16(const BwdParams& p, const CUtensorMap& tmX,
