@@ -1128,8 +1128,10 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
     // ---------------------------------------------------------------- Gaussian warps (4)
     // Warp w owns tile rows 32w..32w+31 and lane l the feature pair (2l, 2l+1) of every K-block:
     // per stage a lane reads one float4 of coefficients and one 4-byte word of each of its
-    // warp's rows, and keeps one running sum per row; a butterfly over the lanes gives the row
-    // totals at the end of the tile.
+    // warp's rows, and keeps a running pair of sums per row (even and odd features, two FMAs in
+    // one instruction); a butterfly over the lanes gives the row totals at the end of the tile.
+    // These warps hold every X stage until they have read it, so their instruction count per
+    // stage sets how fast stages return to the producer.
     if (kGauss) {                            // (warps 6-9)
       const int gw = warp - 6;
       const int gt = gw * 32 + lane;
@@ -1144,28 +1146,33 @@ k_router_fwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
         const int buf = lt & 1;
         const uint32_t use = static_cast<uint32_t>(lt >> 1);
         if (!mbar_wait(g_empty + buf, (use & 1u) ^ 1u, wc)) break;
-        float acc[32];
+        uint64_t acc2[32];                   // per row: {sum over even features, over odd}
 #pragma unroll
-        for (int r = 0; r < 32; ++r) acc[r] = 0.f;
+        for (int r = 0; r < 32; ++r) acc2[r] = 0ull;
         for (int kb = 0; kb < n_kb; ++kb) {
           // the coefficients of this block's chunk (complete for every later tile)
           if (lt == 0 && (kb & 7) == 0 && kb < 8 * kCoefBars &&
               !mbar_wait(coef_bar + (kb >> 3), 0, wc)) { ok = false; break; }
           if (!mbar_wait(full + st, ph, wc)) { ok = false; break; }
           const uint8_t* xs = stage + st * sbytes + gw * 32 * 128;
-          const float4 cf = cq[kb_at(kb) * 32 + lane];
+          // {a_2l, a_2l+1} and {b_2l, b_2l+1} of the float4 {ga, ga, gb, gb}
+          const ulonglong2 cf = reinterpret_cast<const ulonglong2*>(cq)[kb_at(kb) * 32 + lane];
 #pragma unroll
           for (int r = 0; r < 32; ++r) {
             const uint32_t u = *reinterpret_cast<const uint32_t*>(xs + r * 128 + ((chk ^ (r & 7)) << 4) + wcol);
-            const float x0 = __uint_as_float(u << 16), x1 = __uint_as_float(u & 0xffff0000u);
-            acc[r] = fmaf(x0, fmaf(cf.x, x0, cf.z), acc[r]);
-            acc[r] = fmaf(x1, fmaf(cf.y, x1, cf.w), acc[r]);
+            // {x_2l, x_2l+1} widened from the bf16 pair
+            const uint64_t x2 = (static_cast<uint64_t>(u & 0xffff0000u) << 32) | static_cast<uint32_t>(u << 16);
+            acc2[r] = ffma2(x2, ffma2(x2, cf.x, cf.y), acc2[r]);    // x (a x + b) + acc, per half
           }
           __syncwarp();
           if (lane == 0) mbar_arrive(empty + st);
           if (++st == n_stages) { st = 0; ph ^= 1u; }
         }
         if (!ok) break;
+        float acc[32];
+#pragma unroll
+        for (int r = 0; r < 32; ++r)
+          acc[r] = __uint_as_float(static_cast<uint32_t>(acc2[r])) + __uint_as_float(static_cast<uint32_t>(acc2[r] >> 32));
         dll_s[buf * 128 + gt] = warp_transpose_sum(acc);
         mbar_arrive(g_full + buf);
       }
