@@ -805,6 +805,7 @@ smoes_status smoes_bin_balance(smoes_plan P, const int32_t* topk_idx, float loss
   p.gsave = v.gsave;
   p.topk_idx = topk_idx;
   p.expert_bin = v.expert_bin;
+  p.expert_bin_host = P->expert_bin.data();
   p.scale = loss_scale;
   p.part_h = reinterpret_cast<float*>(b + P->L.bal_h);
   p.part_s = reinterpret_cast<int32_t*>(b + P->L.bal_s);

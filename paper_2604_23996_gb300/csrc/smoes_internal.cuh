@@ -220,6 +220,7 @@ struct BalParams {
   const float* gsave;
   const int32_t* topk_idx;
   const int32_t* expert_bin;
+  const int32_t* expert_bin_host;   // the plan's bin map on the host (kernel choice)
   double scale;
   float* part_h;
   int32_t* part_s;
