@@ -9,8 +9,8 @@
 //   sum (x - mu_T)^2 = s2 - s1^2 / n,   mu_T = c + s1 / n,
 // loses nothing to cancellation. k_stats_partial streams X once (16-byte loads, 8 features per
 // thread, fp32 sums over a contiguous run of rows per block) and writes one partial per block;
-// k_stats_finalize sums the partials in block order in fp64 and applies eqs. (5)-(7), also in
-// fp64. Both are deterministic.
+// k_stats_finalize sums the partials in block order (runs of 8 in fp32, then fp64) and applies
+// eqs. (5)-(7) in fp64. Both are deterministic.
 //
 // Adaptive binning. k_adaptive_bins (one block, E <= 256 threads) updates the EMA expert loads
 // of eq. (10) from this step's per-modality selection counts, forms the text bias f_spec of
@@ -151,8 +151,9 @@ __global__ void __launch_bounds__(kStatThreads) k_stats_partial(const StatsParam
 }
 
 // One (modality, feature) column per (block column, 8 slices): slice t sums the partials of
-// blocks [t G / 8, (t+1) G / 8) in order, the slices are added in slice order, all in fp64;
-// then eqs. (5)-(7). The counts |T_m| are summed per block from nvis (in block order).
+// blocks [t G / 8, (t+1) G / 8) in order (runs of 8 in fp32, the runs in fp64), the slices are
+// added in slice order in fp64; then eqs. (5)-(7) in fp64. The counts |T_m| are integer sums of
+// nvis.
 constexpr int kFinSlices = 8;
 constexpr int kFinCols = 32;
 
@@ -166,18 +167,36 @@ __global__ void __launch_bounds__(kFinSlices * kFinCols) k_stats_finalize(const 
   const int m = i2 < 2 * p.d ? i2 / p.d : 0;
   const int i = i2 < 2 * p.d ? i2 % p.d : 0;
   const int G = p.G;
-  if (threadIdx.x == 0) {
+  if (threadIdx.x < 32) {                         // |T_v|: integer counts, lanes stride the blocks
     long long nvis = 0;
-    for (int g = 0; g < G; ++g) nvis += p.nvis[g];
-    cnt_s = nvis;
+    for (int g = threadIdx.x; g < G; g += 32) nvis += p.nvis[g];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) nvis += __shfl_xor_sync(0xffffffffu, nvis, o);
+    if (threadIdx.x == 0) cnt_s = nvis;
   }
+  // runs of 8 block partials added in fp32 (their loads issued together), the runs in fp64: GB300's
+  // fp64 rate is a small fraction of its fp32 rate, and one fp64 add per partial set this
+  // kernel's time
   double a1 = 0.0, a2 = 0.0;
   if (i2 < 2 * p.d) {
     const int g0 = sl * G / kFinSlices, g1 = (sl + 1) * G / kFinSlices;
-    for (int g = g0; g < g1; ++g) {
-      const float* base = p.part + static_cast<size_t>(g) * 4 * p.d;
-      a1 += static_cast<double>(__ldcg(base + static_cast<size_t>(2 * m) * p.d + i));
-      a2 += static_cast<double>(__ldcg(base + static_cast<size_t>(2 * m + 1) * p.d + i));
+    for (int g = g0; g < g1; g += 8) {
+      float v1[8], v2[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const bool in = g + u < g1;
+        const float* base = p.part + static_cast<size_t>(in ? g + u : g0) * 4 * p.d;
+        v1[u] = in ? __ldcg(base + static_cast<size_t>(2 * m) * p.d + i) : 0.f;
+        v2[u] = in ? __ldcg(base + static_cast<size_t>(2 * m + 1) * p.d + i) : 0.f;
+      }
+      float r1 = 0.f, r2 = 0.f;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        r1 += v1[u];
+        r2 += v2[u];
+      }
+      a1 += static_cast<double>(r1);
+      a2 += static_cast<double>(r2);
     }
   }
   red[0][sl][col] = a1;
