@@ -50,4 +50,21 @@ __device__ __forceinline__ float sigmoid_acc(float y) {
   return e / (1.f + e);
 }
 
+// Transpose-reduce of 32 values per lane: afterwards v[0] of lane l holds the sum over the 32
+// lanes of their v[l] (a fixed butterfly tree, 31 shuffles).
+__device__ __forceinline__ float warp_transpose_sum(float (&v)[32]) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int s = 16; s >= 1; s >>= 1) {
+    const bool upper = (lane & s) != 0;
+#pragma unroll
+    for (int i = 0; i < s; ++i) {
+      const float send = upper ? v[i] : v[i + s];
+      const float keep = upper ? v[i + s] : v[i];
+      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
+    }
+  }
+  return v[0];
+}
+
 }  // namespace smoes

@@ -72,23 +72,6 @@ __device__ __noinline__ float gauss_coef_pair(float2 mv, float2 mt, float2 vv, f
   return (g0 && g1) ? c0 + c1 : CUDART_NAN_F;
 }
 
-// Transpose-reduce of 32 values per lane: afterwards v[0] of lane l holds the sum over the 32
-// lanes of their v[l] (a fixed butterfly tree, 31 shuffles).
-__device__ __forceinline__ float warp_transpose_sum(float (&v)[32]) {
-  const int lane = threadIdx.x & 31;
-#pragma unroll
-  for (int s = 16; s >= 1; s >>= 1) {
-    const bool upper = (lane & s) != 0;
-#pragma unroll
-    for (int i = 0; i < s; ++i) {
-      const float send = upper ? v[i] : v[i + s];
-      const float keep = upper ? v[i + s] : v[i];
-      v[i] = keep + __shfl_xor_sync(0xffffffffu, send, s);
-    }
-  }
-  return v[0];
-}
-
 // Reduces sample s (called by the one warp that completed its last piece): fixed-order sums of
 // the pieces, then eqs. (12)-(14) and the backward coefficients
 //   a_k = dI/dSbar_vk / (N_B A_v), b_k = dI/dSbar_tk / (N_B A_t), h_k = (a_k + b_k) / 2,
