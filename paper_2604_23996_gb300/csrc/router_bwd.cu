@@ -11,8 +11,13 @@
 // (dz = hi + lo to ~2^-17 relative) directly in the 128-byte-swizzled shared-memory image the
 // tensor cores read. The main kernel runs CTA (token group g, d-slice s): per tile it bulk-copies
 // that image, and one thread issues, per 128-column d-block of the slice,
-//   dW^T[d-block] += X^T(tile) . dz        (M = 128 d, N = E_pad, K = 64 tokens)  -> TMEM, kept
-//   dX^T[d-block]  = W^T(d-block) . dz^T   (M = 128 d, N = 64 tokens, K = E_pad)  -> TMEM, drained
+//   dW^T[d-block] += X^T(tile) . (hi + lo)  (M = 128 d, N = E_pad, K = 64 tokens)  -> TMEM, kept
+//   dX^T[d-block]  = W^T(d-block) . hi^T    (M = 128 d, N = 64 tokens, K = E_pad)  -> TMEM, drained
+// dW (fp32 output, sums over many tokens that cancel) takes both halves; dX, stored in bf16, is
+// formed from the bf16-rounded dz alone (bf16 inputs, fp32 accumulation: each element within one
+// bf16 ulp plus 2^-8 sum_e |dz_je W_ed| of the exact value). The tensor pipe, not memory, set the
+// tile rate with the lo half in dX as well: its 64-token MMAs read 6 KB of operands for 128 x 64 x
+// 16 products.
 // X tiles arrive by TMA; the W slice stays resident in shared memory; dX leaves by TMA store.
 // The per-group dW^T slice is written once at the end and summed over groups in fixed order.
 #include <cuda_bf16.h>
@@ -502,9 +507,7 @@ k_router_bwd_tc(const __grid_constant__ CUtensorMap tmX, const __grid_constant__
               const uint64_t da = sdesc_sw128(wa + ke * 2048, dz_half, 1024);
               const uint32_t boff = (ke >> 2) * 8192 + (ke & 3) * 32;
               const uint64_t dh = sdesc_sw128(hi + boff, 16, 1024);
-              const uint64_t dl = sdesc_sw128(lo + boff, 16, 1024);
               umma_bf16(dxc, da, dh, id_dx, ke > 0 ? 1u : 0u);
-              umma_bf16(dxc, da, dl, id_dx, 1u);
             }
             umma_commit(dx_full + xb);
           }
