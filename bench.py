@@ -203,16 +203,31 @@ class ClockSampler:
         return out
 
 
-def profile_traffic(kernel_file, workload, call):
+# the sources whose code a call's kernels are compiled from (a traffic record counts only for them)
+TRAFFIC_SOURCES = {
+    "fwd": ["router_fwd.cu", "router_fwd_tc.cuh", "router_fwd_var.cu", "ptx.cuh", "device_common.cuh",
+            "smoes_internal.cuh"],
+    "bwd": ["router_bwd.cu", "ptx.cuh", "device_common.cuh", "smoes_internal.cuh"],
+}
+
+
+def sources_sha(files):
+    """First 16 hex digits of the sha256 of the files' bytes, in order."""
+    h = hashlib.sha256()
+    for name in files:
+        with open(os.path.join(ROOT, "paper_2604_23996_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profile_traffic(kernel_files, workload, call):
     """DRAM bytes per launch of a call (fwd / bwd) from a committed ncu summary, if it was taken on
-    the current source."""
+    the current sources."""
     path = os.path.join(ROOT, "profiles", f"traffic_{workload}_{call}.json")
-    src = os.path.join(ROOT, "paper_2604_23996_gb300", "csrc", kernel_file)
     try:
         with open(path) as f:
             rec = json.load(f)
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        if rec.get("source_sha") == sha:
+        if rec.get("source_sha") == sources_sha(kernel_files):
             return float(rec["dram_bytes_per_launch"])
     except Exception:
         pass
@@ -817,7 +832,7 @@ def main():
             tkey = args.config if args.tokens is None else f"{args.config}_T{wl.T}"
             rooflines[name] = {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
                                "frac": ach / hbm, "bytes": by,
-                               "traffic": profile_traffic(f"router_{call}.cu", tkey, call),
+                               "traffic": profile_traffic(TRAFFIC_SOURCES[call], tkey, call),
                                "kernel": kern, "peak_source": peak_kind + " (burst copy)"}
     dominant = max(t_part, key=lambda n: float(np.mean(t_part[n])))
     line = {

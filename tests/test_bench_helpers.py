@@ -34,11 +34,16 @@ def test_traffic_record_only_for_its_source(tmp_path, monkeypatch):
     prof.mkdir()
     src_dir.mkdir(parents=True)
     src = src_dir / "router_fwd.cu"
+    hdr = src_dir / "router_fwd_tc.cuh"
     src.write_text("// kernel v1\n")
-    sha = hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    hdr.write_text("// header v1\n")
+    sha = hashlib.sha256(src.read_bytes() + hdr.read_bytes()).hexdigest()[:16]
     (prof / "traffic_w_fwd.json").write_text(json.dumps({"source_sha": sha, "dram_bytes_per_launch": 123.0}))
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.profile_traffic("router_fwd.cu", "w", "fwd") == 123.0
-    src.write_text("// kernel v2\n")                      # the kernel changed since the capture
-    assert bench.profile_traffic("router_fwd.cu", "w", "fwd") is None
-    assert bench.profile_traffic("router_fwd.cu", "other", "fwd") is None
+    files = ["router_fwd.cu", "router_fwd_tc.cuh"]
+    assert bench.profile_traffic(files, "w", "fwd") == 123.0
+    hdr.write_text("// header v2\n")                     # a source of the kernel changed since
+    assert bench.profile_traffic(files, "w", "fwd") is None
+    hdr.write_text("// header v1\n")
+    assert bench.profile_traffic(files, "other", "fwd") is None
+    assert bench.profile_traffic(["router_fwd.cu"], "w", "fwd") is None   # a different source set
