@@ -612,6 +612,38 @@ def run_e2e(st, args, world, dev, rate_of):
             "note": "inputs of step i+1 copied while step i computes (two device buffers)"}
 
 
+def dedup_report(st):
+    """Expert-parallel transfer ratios of the step's dispatch (Sec. 4.5), from the permutation the
+    GPU produced: with the bins as devices and a token's home device floor(j K / T) (a contiguous
+    data-parallel split), w/o DeDup = remote (token, expert) selections / (T k), w/ DeDup = remote
+    unique (token, bin) pairs / T. The dispatch matrix gives the second directly."""
+    import torch
+    r, wl = st.r, st.wl
+    if torch.cuda.is_available():
+        torch.cuda.synchronize()
+    T, K, k = wl.T, wl.n_bins, wl.k
+    D = r.dispatch.cpu().numpy().astype(np.int64)                 # [home, bin] unique pairs
+    off = r.bin_offsets.cpu().numpy().astype(np.int64)
+    P = int(off[-1])
+    tok = r.perm_token[:P].cpu().numpy().astype(np.int64)
+    mask = r.perm_mask[:P].cpu().numpy().view(np.uint32).astype(np.uint64)
+    b = np.repeat(np.arange(K), np.diff(off))
+    home = (tok * K) // T
+    sel = np.zeros(P, dtype=np.int64)                             # selected experts per entry
+    m = mask.copy()
+    while np.any(m):
+        sel += (m & 1).astype(np.int64)
+        m >>= np.uint64(1)
+    remote_pairs = int(D.sum() - np.trace(D))
+    remote_sel = int(sel[home != b].sum())
+    return {"home": "floor(j K / T)", "devices": K,
+            "ratio_without_dedup": remote_sel / float(T * k),
+            "ratio_with_dedup": remote_pairs / float(T),
+            "unique_pairs_per_token": P / float(T),
+            "check": "remote pairs from the dispatch matrix = remote entries of the permutation: "
+                     + str(remote_pairs == int((home != b).sum()))}
+
+
 def graph_time(fn, steps, flush):
     """Mean device time (ms) of fn replayed from a CUDA graph, L2 flushed before each replay."""
     import torch
@@ -853,6 +885,7 @@ def main():
     }
     if sweep is not None:
         line["sweep"] = sweep
+    line["dedup"] = dedup_report(st)
     if nxt is not None:
         line["next_rows"] = nxt
     if not args.no_cpu_baseline and world == 1:

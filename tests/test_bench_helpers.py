@@ -1,11 +1,12 @@
 """Host-side arithmetic of bench.py (no GPU): the algorithmic bytes and flops behind the
-roofline fractions, and the rule that an ncu traffic record counts only for the source it was
-taken on."""
+roofline fractions, the rule that an ncu traffic record counts only for the sources it was
+taken on, and the expert-parallel transfer ratios derived from a dispatch."""
 import hashlib
 import json
 import os
 import sys
 
+import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -47,3 +48,31 @@ def test_traffic_record_only_for_its_source(tmp_path, monkeypatch):
     hdr.write_text("// header v1\n")
     assert bench.profile_traffic(files, "other", "fwd") is None
     assert bench.profile_traffic(["router_fwd.cu"], "w", "fwd") is None   # a different source set
+
+
+def test_dedup_report_counts_remote_transfers():
+    # a tiny dispatch through the oracle's permutation, read back by the bench's report, against a
+    # brute-force count over the (token, expert) selections with home(j) = floor(j K / T)
+    from types import SimpleNamespace
+
+    import torch
+
+    from oracle import smoes_oracle as O
+    rng = np.random.default_rng(3)
+    T, E, k, K = 37, 12, 3, 4
+    eb = np.arange(E) // (E // K)
+    topk = np.stack([rng.choice(E, k, replace=False) for _ in range(T)]).astype(np.int32)
+    pr = O.bin_permute(topk, eb, K)
+    r = SimpleNamespace(dispatch=torch.from_numpy(pr["dispatch"].astype(np.int32)),
+                        bin_offsets=torch.from_numpy(pr["offsets"].astype(np.int32)),
+                        perm_token=torch.from_numpy(pr["perm"].astype(np.int32)),
+                        perm_mask=torch.from_numpy(pr["mask"].astype(np.uint32).view(np.int32)))
+    st = SimpleNamespace(r=r, wl=SimpleNamespace(T=T, n_bins=K, k=k))
+    rep = bench.dedup_report(st)
+    home = (np.arange(T) * K) // T
+    remote_sel = sum(int(eb[e] != home[j]) for j in range(T) for e in topk[j])
+    remote_pairs = sum(len({int(eb[e]) for e in topk[j]} - {int(home[j])}) for j in range(T))
+    assert rep["ratio_without_dedup"] == remote_sel / (T * k)
+    assert rep["ratio_with_dedup"] == remote_pairs / T
+    assert rep["check"].endswith("True")
+    assert rep["ratio_with_dedup"] <= rep["ratio_without_dedup"] * k
