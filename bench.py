@@ -616,7 +616,8 @@ def dedup_report(st):
     """Expert-parallel transfer ratios of the step's dispatch (Sec. 4.5), from the permutation the
     GPU produced: with the bins as devices and a token's home device floor(j K / T) (a contiguous
     data-parallel split), w/o DeDup = remote (token, expert) selections / (T k), w/ DeDup = remote
-    unique (token, bin) pairs / T. The dispatch matrix gives the second directly."""
+    unique (token, bin) pairs / T (also per selection, / (T k), and the share of remote copies
+    that DeDup saves). The dispatch matrix gives the remote pairs directly."""
     import torch
     r, wl = st.r, st.wl
     if torch.cuda.is_available():
@@ -639,6 +640,8 @@ def dedup_report(st):
     return {"home": "floor(j K / T)", "devices": K,
             "ratio_without_dedup": remote_sel / float(T * k),
             "ratio_with_dedup": remote_pairs / float(T),
+            "ratio_with_dedup_per_selection": remote_pairs / float(T * k),
+            "dedup_saving": 1.0 - remote_pairs / float(remote_sel) if remote_sel else 0.0,
             "unique_pairs_per_token": P / float(T),
             "check": "remote pairs from the dispatch matrix = remote entries of the permutation: "
                      + str(remote_pairs == int((home != b).sum()))}

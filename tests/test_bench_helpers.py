@@ -74,5 +74,7 @@ def test_dedup_report_counts_remote_transfers():
     remote_pairs = sum(len({int(eb[e]) for e in topk[j]} - {int(home[j])}) for j in range(T))
     assert rep["ratio_without_dedup"] == remote_sel / (T * k)
     assert rep["ratio_with_dedup"] == remote_pairs / T
+    assert rep["ratio_with_dedup_per_selection"] == remote_pairs / (T * k)
+    assert rep["dedup_saving"] == 1.0 - remote_pairs / remote_sel
     assert rep["check"].endswith("True")
     assert rep["ratio_with_dedup"] <= rep["ratio_without_dedup"] * k
