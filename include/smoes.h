@@ -254,7 +254,9 @@ smoes_status smoes_router_fwd_permute(smoes_plan plan, const void* X, const void
  *   tensors of the preceding smoes_router_fwd on the same ws.
  *   dW [E, d] float32: written, or accumulated into when accumulate_dW != 0.
  *   dX [T, d] (plan dtype) or NULL; dlogits [T, E] float32 or NULL.
- *   d_topk_w [T, k] float32 or NULL. */
+ *   d_topk_w [T, k] float32 or NULL.
+ *   Precision on SMOES_BF16 plans: dW is formed from dz split into two bf16 parts (fp32-level
+ *   accuracy); dX from dz rounded to bf16 (bf16 inputs, fp32 accumulation), stored in bf16. */
 smoes_status smoes_router_bwd(smoes_plan plan, const void* X, const void* W, const float* M,
                               const int32_t* topk_idx, const float* d_topk_w, float loss_scale,
                               float* dW, int accumulate_dW, void* dX, float* dlogits,
@@ -270,7 +272,7 @@ smoes_status smoes_router_bwd(smoes_plan plan, const void* X, const void* W, con
  *   next forward adds the gradient of loss_scale * L_bal, taken with the counts f_e constant, to
  *   the MI gradient (dlogits, dW and dX; topk_idx must then be passed to smoes_router_bwd). The
  *   arming is tracked both on the host (the plan) and in ws (the forward kernels clear it).
- *   Sums are fp32 per block of tokens and fp64 across blocks, in a fixed order. */
+ *   Sums are fp32, in a fixed order (bitwise reproducible). */
 smoes_status smoes_bin_balance(smoes_plan plan, const int32_t* topk_idx, float loss_scale,
                                float* loss_bal, float* f_e, float* P_e, void* ws, size_t ws_bytes,
                                cudaStream_t stream);
