@@ -106,7 +106,8 @@ def workload_text(config, wl):
 
 
 def bench_config(config, wl, world):
-    """The `config` object of the JSON line; both arms print the same one."""
+    """The `config` object of the JSON line. Both arms print the same workload; the reference arm
+    replaces the two keys that describe how the device is timed."""
     use_attn = config == "attn_router"
     return {"workload": f"{config}: {workload_text(config, wl)}; "
                         + (f"attention score ({wl.B if wl is not None else 8}x4096, 16 heads, hd 128, "
@@ -359,7 +360,10 @@ def run_reference(args, rank, world):
             "warmup": args.warmup, "ms_per_step": 1e3 * t_tot / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
-            "config": bench_config(args.config, wl, world),
+            "config": dict(bench_config(args.config, wl, world),
+                           l2="not applicable (host cores)",
+                           timing="host wall clock (time.perf_counter) around each sample's "
+                                  "oracle evaluation"),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle",
                              "cpu_model": cpu_model(),
                              "sample": f"the whole batch ({wl.B} samples, {wl.T} tokens) per step; "
