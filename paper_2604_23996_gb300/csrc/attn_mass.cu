@@ -14,8 +14,9 @@
 // order). Sixteen softmax warps keep the special-function unit, which evaluates one
 // exponential per score, busier than eight could. The head's score a / l goes to the workspace;
 // the last head of each (sequence, query tile) to finish averages the heads in fixed order and
-// writes M (optionally blended with the carried score by eq. 4). Items are handed out longest
-// first so that the CTAs finish together.
+// writes M (optionally blended with the carried score by eq. 4). Items are ordered longest
+// first and dealt to the CTAs in rounds of alternating direction, so that the CTAs finish
+// together.
 #include <cuda_bf16.h>
 #include <math_constants.h>
 
@@ -44,7 +45,7 @@ __host__ __device__ inline AttnLayout attn_layout(int n_ks) {
   L.k = o;    o += static_cast<uint32_t>(n_ks) * kTile;    // K blocks
   L.mk = o;   o += 4u * 2u * 2u * kHalf * 4u;              // bias*log2e [64] | m [64]: group x buffer
   L.mrg = o;  o += 2u * 2u * 3u * kAT * 4u;                // second half's (max, l, a): tile x buffer
-  L.bars = o; o += 8u * (2u * n_ks + 30u) + 32u;
+  L.bars = o; o += 8u * (2u * n_ks + 36u) + 32u;
   L.total = o + 1024u;
   return L;
 }
@@ -72,6 +73,15 @@ __device__ __forceinline__ void add2(float& d0, float& d1, float a0, float a1, f
       "add.rn.f32x2 rd, ra, rb;\n\t"
       "mov.b64 {%0, %1}, rd;\n\t}"
       : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
+// Bounded wait with its slow path out of line: the softmax warps keep the wait context in
+// memory instead of in registers, which their 96-register budget needs for the scores.
+__device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, const WaitCtx& w) {
+  return mbar_wait(bar, parity, w);
+}
+__device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, const WaitCtx& w) {
+  return mbar_try_wait(bar, parity) || wait_slow(bar, parity, w);
 }
 
 // Work item -> (sequence b, head h, query-tile pair pr). Pairs run longest (last) first; within
@@ -120,9 +130,10 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
   uint64_t* mk_bar = q_full + 12;       // [group][buf] keys' (bias, m) staged by that group
   uint64_t* out_bar = q_full + 20;      // [tile] head results of the tile written
   uint64_t* dec_bar = q_full + 22;      // [tile] the ticket decision of the tile is published
-  uint64_t* mrg_bar = q_full + 24;      // [tile] the second half's state of the item is written
-  uint64_t* drain = q_full + 26;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 28);
+  uint64_t* mrg_full = q_full + 24;     // [tile][merge buffer] the second half's state is written
+  uint64_t* mrg_free = q_full + 28;     // [tile][merge buffer] the first half has read it
+  uint64_t* drain = q_full + 32;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(q_full + 34);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
   volatile uint32_t* decision = reinterpret_cast<volatile uint32_t*>(tmem_slot + 2);   // [2]
 
@@ -141,7 +152,10 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       mbar_init(q_empty + t, 1);
       mbar_init(out_bar + t, 128);
       mbar_init(dec_bar + t, 1);
-      mbar_init(mrg_bar + t, 128);
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(mrg_full + 2 * t + i, 128);
+        mbar_init(mrg_free + 2 * t + i, 128);
+      }
       for (int i = 0; i < 2; ++i) {
         mbar_init(s_full + 2 * t + i, 1);
         mbar_init(s_empty + 2 * t + i, 256);     // both key halves read the scores
@@ -169,7 +183,9 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       int nqt[2] = {0, 0};              // items that used Q buffer t: its barrier phase
       long issued = 0;
       bool ok = true;
-      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      for (int rd = 0; ok; ++rd) {
+        const int item = dealt_item(rd);
+        if (item >= n_items) break;
         const Item w = decode_item(p, item);
         const int row0 = (w.b * p.H + w.h) * p.S;
         for (int t = 0; t < w.nq && ok; ++t) {
@@ -209,7 +225,9 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       int blk[2] = {0, 0};              // running block count per tile: selects its TMEM buffer
       int nqt[2] = {0, 0};
       bool ok = true;
-      for (int item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      for (int rd = 0; ok; ++rd) {
+        const int item = dealt_item(rd);
+        if (item >= n_items) break;
         const Item w = decode_item(p, item);
         for (int t = 0; t < w.nq && ok; ++t)
           if (!mbar_wait(q_full + t, static_cast<uint32_t>(nqt[t]++) & 1u, wc)) ok = false;
@@ -267,7 +285,9 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
     uint64_t* mkbar = mk_bar + 2 * grp;
     int blk = 0;
     int ng = 0;                                // items this group has processed
-    for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
+    for (int rd = 0; ; ++rd) {
+      const int item = dealt_item(rd);
+      if (item >= n_items) break;
       const Item w = decode_item(p, item);
       if (t >= w.nq) continue;
       const int qt = w.qt0 + t;
@@ -299,8 +319,8 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         }
         mbar_arrive(mkbar + buf);
         if (kb + 1 < nkb) key_vals(kb + 1, nb_bias, nb_m);
-        if (!mbar_wait(mkbar + buf, use & 1u, wc)) { ok = false; break; }
-        if (!mbar_wait(sfull + buf, use & 1u, wc)) { ok = false; break; }
+        if (!wait_bar(mkbar + buf, use & 1u, wc)) { ok = false; break; }
+        if (!wait_bar(sfull + buf, use & 1u, wc)) { ok = false; break; }
         tc_fence_after();
         const uint32_t ta = tmem + (static_cast<uint32_t>(lg * 32) << 16) + static_cast<uint32_t>((2 * t + buf) * kAT);
         const float4* bias4 = reinterpret_cast<const float4*>(mkg + buf * kAT);
@@ -361,18 +381,26 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       float l = (l4[0] + l4[1]) + (l4[2] + l4[3]);
       float a = (a4[0] + a4[1]) + (a4[2] + a4[3]);
       const uint32_t nt = static_cast<uint32_t>(ng++);   // this item's phase of the group's barriers
-      // the second half hands its state to the first, which merges it (maxima in log2 units)
-      float* mb = mrt + (nt & 1u) * 3 * kAT;
+      // the second half hands its state to the first, which merges it (maxima in log2 units).
+      // Two merge buffers alternate by item; the second half may run ahead of the first by up
+      // to two S buffers of keys, which can span whole short items, so it refills a buffer only
+      // once the first half has read the buffer's previous state (full / free pair per buffer).
+      const uint32_t mbuf = nt & 1u, muse = nt >> 1;
+      float* mb = mrt + mbuf * 3 * kAT;
+      uint64_t* mfull = mrg_full + 2 * t + mbuf;
+      uint64_t* mfree = mrg_free + 2 * t + mbuf;
       if (hf == 1) {
+        if (!wait_bar(mfree, (muse & 1u) ^ 1u, wc)) break;
         mb[row] = mrun;
         mb[kAT + row] = l;
         mb[2 * kAT + row] = a;
-        mbar_arrive(mrg_bar + t);
+        mbar_arrive(mfull);
         continue;
       }
-      if (!mbar_wait(mrg_bar + t, nt & 1u, wc)) break;
+      if (!wait_bar(mfull, muse & 1u, wc)) break;
       {
         const float m1 = mb[row], l1 = mb[kAT + row], a1 = mb[2 * kAT + row];
+        mbar_arrive(mfree);
         const float mm = fmaxf(mrun, m1);
         if (mm == -CUDART_INF_F) {
           l = 0.f;
@@ -391,7 +419,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
       mbar_arrive(out_bar + t);
       if (gt == 0) {
         uint32_t last = 0u;
-        if (mbar_wait(out_bar + t, nt & 1u, wc)) {
+        if (wait_bar(out_bar + t, nt & 1u, wc)) {
           const uint32_t n = atomicAdd(p.ticket + w.b * p.n_qtiles + qt, 1u) + 1u;
           last = (n == static_cast<uint32_t>(p.H)) ? 1u : 0u;
           if (last) p.ticket[w.b * p.n_qtiles + qt] = 0u;     // ready for the next call
@@ -399,7 +427,7 @@ k_attn_mass(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUt
         decision[t] = last;
         mbar_arrive(dec_bar + t);
       }
-      if (!mbar_wait(dec_bar + t, nt & 1u, wc)) break;
+      if (!wait_bar(dec_bar + t, nt & 1u, wc)) break;
       if (decision[t] && valid) {
         __threadfence();
         float sum = 0.f;

@@ -2,7 +2,9 @@
 
 Cases: sequence lengths that are not multiples of the 128-query tile, causal and non-causal
 attention, a vision-key logit bias, hard labels (eq. 2) and a carried soft score, the eq. (4)
-residual blend, and short sequences (S < 128).
+residual blend, short sequences (S < 128), and many short work items per CTA (320 (sequence,
+head) items of one or two key blocks on 152 CTAs: the second key half of a CTA can run a whole
+item ahead of the first, which the merge hand-off between the halves has to absorb).
 """
 import numpy as np
 import pytest
@@ -63,6 +65,7 @@ def _run(bd, Q, K, is_vis, m, key_bias, causal, soft, norms=None):
     (2, 2, 200, False, False),
     (3, 4, 77, True, False),
     (1, 16, 1024, True, False),
+    (20, 16, 256, True, False),
 ])
 def test_attention_mass_parity(bd, B, H, S, causal, soft):
     Q, K, is_vis, m, key_bias = _case(B * 100 + S, B, H, S, soft=soft)
