@@ -75,6 +75,15 @@ __device__ __forceinline__ void add2(float& d0, float& d1, float a0, float a1, f
       : "=f"(d0), "=f"(d1) : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 
+// Work items of a persistent kernel, dealt to the CTAs in rounds of gridDim.x that alternate in
+// direction: in round r CTA c takes item r * G + c when r is even and r * G + (G - 1 - c) when it
+// is odd. With the items ordered longest first, each CTA's total stays within about one item of
+// the mean, where a plain stride gives the low-numbered CTAs the longest item of every round.
+__device__ __forceinline__ int dealt_item(int round) {
+  const int g = static_cast<int>(gridDim.x), c = static_cast<int>(blockIdx.x);
+  return round * g + ((round & 1) ? g - 1 - c : c);
+}
+
 // Bounded wait with its slow path out of line: the softmax warps keep the wait context in
 // memory instead of in registers, which their 96-register budget needs for the scores.
 __device__ __noinline__ bool wait_slow(uint64_t* bar, uint32_t parity, const WaitCtx& w) {

@@ -67,13 +67,4 @@ __device__ __forceinline__ float warp_transpose_sum(float (&v)[32]) {
   return v[0];
 }
 
-// Work items of a persistent kernel, dealt to the CTAs in rounds of gridDim.x that alternate in
-// direction: in round r CTA c takes item r * G + c when r is even and r * G + (G - 1 - c) when it
-// is odd. With the items ordered longest first, each CTA's total stays within about one item of
-// the mean, where a plain stride gives the low-numbered CTAs the longest item of every round.
-__device__ __forceinline__ int dealt_item(int round) {
-  const int g = static_cast<int>(gridDim.x), c = static_cast<int>(blockIdx.x);
-  return round * g + ((round & 1) ? g - 1 - c : c);
-}
-
 }  // namespace smoes
