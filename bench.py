@@ -120,6 +120,13 @@ def bench_config(config, wl, world):
             "parallelism": f"replicas x{world}"}
 
 
+
+def reference_config(config, wl, world):
+    """The reference arm's `config`: our arm's workload and parallelism, with the two keys that
+    describe the device timing replaced by how the oracle is timed."""
+    return dict(bench_config(config, wl, world), l2="not applicable (host cores)",
+                timing="host wall clock (time.perf_counter) around each sample's oracle evaluation")
+
 def algorithmic(wl):
     """Algorithmic bytes and flops of one step, and bytes of its forward and backward calls."""
     T, d, E, k, K = wl.T, wl.d, wl.E, wl.k, wl.n_bins
@@ -360,10 +367,7 @@ def run_reference(args, rank, world):
             "warmup": args.warmup, "ms_per_step": 1e3 * t_tot / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "impl": "reference",
-            "config": dict(bench_config(args.config, wl, world),
-                           l2="not applicable (host cores)",
-                           timing="host wall clock (time.perf_counter) around each sample's "
-                                  "oracle evaluation"),
+            "config": reference_config(args.config, wl, world),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores(), "kind": "oracle",
                              "cpu_model": cpu_model(),
                              "sample": f"the whole batch ({wl.B} samples, {wl.T} tokens) per step; "

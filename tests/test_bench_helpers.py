@@ -78,3 +78,12 @@ def test_dedup_report_counts_remote_transfers():
     assert rep["dedup_saving"] == 1.0 - remote_pairs / remote_sel
     assert rep["check"].endswith("True")
     assert rep["ratio_with_dedup"] <= rep["ratio_without_dedup"] * k
+
+
+def test_reference_arm_config_names_the_same_workload():
+    wl = config_workload("tiny_fp32")
+    ours = bench.bench_config("tiny_fp32", wl, 1)
+    ref = bench.reference_config("tiny_fp32", wl, 1)
+    assert ref["workload"] == ours["workload"] and ref["parallelism"] == ours["parallelism"]
+    assert "CUDA graph" in ours["timing"] and "host wall clock" in ref["timing"]
+    assert ref["l2"].startswith("not applicable")
